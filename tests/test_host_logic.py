@@ -1,0 +1,75 @@
+"""Host-side logic: input generator and budget schedules (no GPU)."""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2608_23253_gb300 import budget, synth
+from tests.conftest import GOLDEN
+
+
+def test_avg_tokens_printed_schedules():
+    g = json.load(open(os.path.join(GOLDEN, "avg_tokens_schedules.json")))
+    for s in g["schedules"]:
+        got = budget.avg_tokens(g["n_layers"], g["n_visual"], g["prune_after"], s["keep"])
+        assert got == s["avg"], s
+
+
+def test_avg_tokens_layer_spans():
+    t = budget.tokens_per_layer(32, 576, [3, 17, 22], [122, 48, 42])
+    assert t[:3] == [576] * 3 and t[3:17] == [122] * 14 and t[17:22] == [48] * 5 and t[22:] == [42] * 10
+
+
+def test_bf16_rounding_matches_torch():
+    x = np.random.default_rng(0).normal(size=100000).astype(np.float32) * 7
+    x[:4] = [0.0, -0.0, 1.00390625, 1.01171875]      # exact ties to even
+    want = torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(synth.bf16_bits(x), want)
+    assert np.array_equal(synth.bf16_to_f32(want), torch.from_numpy(want.view(np.int16)).view(
+        torch.bfloat16).float().numpy())
+
+
+@pytest.mark.parametrize("cfg", [0, 1, 2, 3, 4])
+def test_config_shapes(cfg):
+    spec = synth.config_spec(cfg)
+    if cfg == 0:
+        assert (spec.B, spec.L, spec.H, spec.images[0].n_text, spec.images[0].keep) == (1, 2, 32, 32, 64)
+    if cfg == 1:
+        assert (spec.B, spec.L, spec.hidden, spec.images[0].n_tok) == (1, 3, 4096, 675)
+    if cfg == 2:
+        nts = [im.n_text for im in spec.images]
+        assert spec.B == 32 and min(nts) >= 16 and max(nts) <= 128 and len(set(nts)) > 5
+    if cfg == 3:
+        assert (spec.H, spec.H_kv, spec.B) == (28, 4, 16)
+        for im in spec.images:
+            assert (im.grid_h, im.grid_w) in [(16, 16), (24, 32), (32, 32), (36, 36)]
+            assert im.keep == {256: 28, 768: 85, 1024: 114, 1296: 144}[im.n_vis]
+    if cfg == 4:
+        assert {im.n_vis: im.keep for im in spec.images} == {2304: 253, 4096: 451}
+        assert {im.n_vis: im.n_salient for im in spec.images} == {2304: 115, 4096: 205}
+
+
+def test_generator_deterministic_and_planted():
+    spec = synth.config_spec(1)
+    a = synth.make_inputs(spec, with_payload=False)
+    b = synth.make_inputs(spec, with_payload=False)
+    assert np.array_equal(a.k, b.k) and np.array_equal(a.q_text, b.q_text)
+    assert a.salient[0].size == 40
+    assert a.k.shape == (3, 675, 32, 128) and a.q_text.shape == (3, 64, 32, 128)
+    k = synth.bf16_to_f32(a.k[0, :, 0]).astype(np.float64)
+    norms = np.linalg.norm(k, axis=1)
+    sal = 35 + a.salient[0]
+    others = np.setdiff1d(np.arange(35, 611), sal)
+    assert norms[sal].mean() > 3 * norms[others].mean()
+
+
+def test_blobs_are_spatially_clustered():
+    spec = synth.config_spec(1)
+    inp = synth.make_inputs(spec, with_payload=False)
+    s = inp.salient[0]
+    i, j = s // 24, s % 24
+    # 40 points in 3 blobs: the mean nearest-neighbour distance is ~1 grid step
+    d = np.sqrt((i[:, None] - i[None]) ** 2 + (j[:, None] - j[None]) ** 2) + np.eye(s.size) * 99
+    assert d.min(axis=1).mean() < 1.5
