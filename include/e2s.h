@@ -1,0 +1,196 @@
+/*
+ * e2s.h -- C ABI of the GB300 (sm_103a) E2S-Pruner pruning decision.
+ *
+ * One pruning step of Algorithm 1 (E2S-Pruner) for a packed batch of images:
+ *
+ *   e2s_score    text-to-visual attention score a[l][h][n]       (Sec. 3.1, Eq. 1)
+ *   e2s_fuse     support, reliability, layer mass, Dempster-Shafer
+ *                fusion across layers, plausibility and priority q (Sec. 4.1-4.2,
+ *                Eqs. 8-19)
+ *   e2s_select   spatial-novelty bonus and global Top-K            (Sec. 4.3, Eqs. 20-23)
+ *   e2s_compact  gather of the retained hidden / K / V rows so that the next
+ *                layer runs on the shortened sequence (Sec. 4, opening
+ *                paragraph; Sec. 5.1.2 pruning settings)
+ *
+ * Conventions shared by every call:
+ *   - Every array argument is a DEVICE pointer unless its comment says host.
+ *     The caller owns all memory, including the workspace; the library never
+ *     allocates and never synchronises (except e2s_read_status).
+ *   - Calls are asynchronous and ordered on the given stream (a cudaStream_t
+ *     passed as void*, NULL = legacy default stream).  They keep no state
+ *     between calls and may be issued from several host threads.
+ *   - The return value reports host-side argument validation and launch
+ *     errors only.  Errors found on the device (inconsistent layout arrays,
+ *     a bounded wait that ran out) are OR-ed into a status word at the start
+ *     of the workspace; e2s_read_status fetches it.
+ *   - bf16 tensors are raw 16-bit bfloat16 patterns.  Results are
+ *     deterministic: reductions run in a fixed order, and ties in the cell
+ *     arg-max and in Top-K go to the lower index.
+ *
+ * Token layout of image b (Sec. 3.1): [system S_b][visual N_V,b on an
+ * h_b x w_b grid, raster order][text N_T,b].  T_b = S_b + N_V,b + N_T,b.
+ * Images are packed back to back; tok_off / vis_off / text_off are the
+ * exclusive prefix sums of T_b / N_V,b / N_T,b (length B+1).
+ */
+#ifndef E2S_H_
+#define E2S_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  E2S_OK = 0,
+  E2S_ERR_INVALID_ARG = 1,   /* null pointer, bad enum value, bad parameter   */
+  E2S_ERR_SHAPE = 2,         /* inconsistent sizes (host or device detected)   */
+  E2S_ERR_ALIGNMENT = 3,     /* pointer or stride not 16-byte aligned          */
+  E2S_ERR_UNSUPPORTED = 4,   /* valid but not implemented (e.g. d != 128)      */
+  E2S_ERR_WORKSPACE = 5,     /* workspace missing, too small or misaligned     */
+  E2S_ERR_CUDA = 6,          /* a CUDA runtime/driver call failed              */
+  E2S_ERR_TIMEOUT = 7        /* a bounded device wait ran out (device status)  */
+} e2s_status;
+
+/* Batch layout.  Pointer members are device arrays of int32. */
+typedef struct {
+  int32_t B;                 /* images in the batch, >= 1                         */
+  int32_t L;                 /* evidence layers, >= 1                             */
+  int32_t H;                 /* query heads                                       */
+  int32_t H_kv;              /* key/value heads; H % H_kv == 0 (GQA group H/H_kv) */
+  int32_t d;                 /* head dimension; 128 is the only supported value   */
+  const int32_t* tok_off;    /* [B+1] packed row offset of image b (K, V, hidden) */
+  const int32_t* n_sys;      /* [B]   S_b                                         */
+  const int32_t* n_vis;      /* [B]   N_V,b = grid_h[b] * grid_w[b]               */
+  const int32_t* n_text;     /* [B]   N_T,b >= 1                                  */
+  const int32_t* grid_h;     /* [B]   visual grid height                          */
+  const int32_t* grid_w;     /* [B]   visual grid width                           */
+  const int32_t* vis_off;    /* [B+1] packed offset into per-visual-token arrays  */
+  const int32_t* text_off;   /* [B+1] packed offset into text-query rows          */
+  int32_t max_T, max_vis, max_text;    /* HOST values: maxima over the batch      */
+  int32_t sum_T, sum_vis, sum_text;    /* HOST values: tok_off[B], vis_off[B], text_off[B] */
+} e2s_layout;
+
+/* Score modes.  EQ1 is Eq. 1 as printed: the mean over text queries of the
+ * pre-softmax logit Q_t K_n / sqrt(d).  CAUSAL_PROB is the attention
+ * probability the model itself computes: softmax of Q_t K^T / sqrt(d) over
+ * the text row's full causal key prefix (keys 0 .. S+N_V+t), visual columns
+ * kept, mean over the text rows. */
+enum { E2S_SCORE_EQ1 = 0, E2S_SCORE_CAUSAL_PROB = 1 };
+
+/* Normalisation of Eq. 8 over the candidate tokens.  DEFAULT = SOFTMAX for
+ * EQ1 and RENORM (r = a / sum a, which keeps r = 1/N_l as "average") for
+ * CAUSAL_PROB, where a softmax of probabilities would be nearly uniform. */
+enum { E2S_NORM_DEFAULT = 0, E2S_NORM_SOFTMAX = 1, E2S_NORM_RENORM = 2 };
+
+/* Flags.  The first five are the ablations of Table 2 (A1-A5). */
+enum {
+  E2S_NO_RELIABILITY = 1u << 0,   /* A2: rho = 1 (Bayesian masses)                      */
+  E2S_NO_LAYER_FUSION = 1u << 1,  /* A3: only the last evidence layer, no prior         */
+  E2S_NO_CONFLICT = 1u << 2,      /* A4: q = Pl                                         */
+  E2S_NO_NOVELTY = 1u << 3,       /* A5: lambda = 0                                     */
+  E2S_VANILLA = 1u << 4,          /* A1: q = mean over layers and heads of a, lambda = 0 */
+  E2S_SIMT_SCORE = 1u << 8        /* e2s_score: plain SIMT kernel instead of tcgen05    */
+};
+
+typedef struct {
+  float lambda;        /* spatial novelty weight, Eq. 22; paper value 0.1         */
+  int32_t G;           /* G x G spatial cells, Sec. 4.3; paper value 4; 1..8      */
+  int32_t score_mode;  /* E2S_SCORE_*                                            */
+  int32_t norm_mode;   /* E2S_NORM_*                                             */
+  uint32_t flags;      /* E2S_* flags                                            */
+} e2s_params;
+
+/* Bytes of workspace every call below needs (status word + per-(image, layer,
+ * head) normalisation statistics).  The workspace must be 256-byte aligned
+ * and its first 4 bytes zero before the first call (see e2s_clear_status). */
+size_t e2s_workspace_size(const e2s_layout* layout, const e2s_params* params);
+
+/* Text-to-visual score (Sec. 3.1, Eq. 1; Algorithm 1 "Compute a_{l,h,n}").
+ *   q_text  bf16 [L][sum_text] rows of (H x d), row stride q_row_stride elements
+ *           (>= H*d, multiple of 8); layer l starts at row l*sum_text.
+ *   k       bf16 [L][sum_T] rows of (H_kv x d), row stride k_row_stride elements
+ *           (>= H_kv*d, multiple of 8); layer l starts at row l*sum_T.
+ *           Query head h uses key head h / (H / H_kv).
+ *   a_out   fp32 [L][H][sum_vis]: a[l][h][vis_off[b] + n].
+ * q_text and k must be 16-byte aligned.  The default path is a tcgen05/TMEM
+ * kernel with TMA-staged K tiles; flag E2S_SIMT_SCORE selects a plain SIMT
+ * kernel with the same results (used to cross-check). */
+e2s_status e2s_score(const e2s_layout* layout, const e2s_params* params,
+                     const void* q_text, int64_t q_row_stride,
+                     const void* k, int64_t k_row_stride,
+                     float* a_out, void* ws, size_t ws_bytes, void* stream);
+
+/* Evidence and fusion (Sec. 4.1-4.2, Eqs. 8-19; Algorithm 1 inner loops).
+ *   a          fp32 [L][H][sum_vis] from e2s_score.
+ *   cand       nullable int32 [sum_vis]: original raster index of visual slot n
+ *              (a later progressive step); NULL = identity.  Only e2s_select
+ *              reads it; accepted here for symmetry and ignored.
+ *   prior      nullable fp32 [sum_vis][4] (m~(I), m~(U), m~(Theta), -): fused
+ *              mass carried from an earlier pruning step.  NULL: the first
+ *              layer initialises the fusion (Eq. 12) and K^(1) = 0.
+ *   mass_out   nullable fp32 [L][sum_vis][4]: (m(I), m(U), m(Theta), p_bar) (Eq. 11).
+ *   fused_out  fp32 [sum_vis][4]: (m~(I), m~(U), m~(Theta), K) after the last layer;
+ *              K is the conflict of the latest combination (Eq. 13).
+ *   q_out      fp32 [sum_vis]: retention priority q (Eq. 19).
+ * Total conflict (1 - K <= 0) gives the vacuous mass (0, 0, 1) and K = 1. */
+e2s_status e2s_fuse(const e2s_layout* layout, const e2s_params* params,
+                    const float* a, const int32_t* cand, const float* prior,
+                    float* mass_out, float* fused_out, float* q_out,
+                    void* ws, size_t ws_bytes, void* stream);
+
+/* Spatial novelty and Top-K (Sec. 4.3, Eqs. 20-23).
+ *   q            fp32 [sum_vis] priorities (e2s_fuse q_out).
+ *   cand         nullable int32 [sum_vis] original raster index of each slot
+ *                (ascending per image); NULL = identity.  Cells follow the
+ *                original grid: cell(i, j) = (i*G/h, j*G/w), integer division.
+ *   keep_count   int32 [B] K_b >= 0.
+ *   keep_off     int32 [B+1] exclusive prefix sum of keep_count.
+ *   sum_keep     HOST int: keep_off[B].
+ *   keep_idx     int32 [sum_keep] out: image-local visual slot indices, ascending
+ *                per image.  If K_b > N_V,b all slots are kept and the spare
+ *                entries are -1.
+ *   q_tilde_out  nullable fp32 [sum_vis]: q~ of Eq. 22. */
+e2s_status e2s_select(const e2s_layout* layout, const e2s_params* params,
+                      const float* q, const int32_t* cand,
+                      const int32_t* keep_count, const int32_t* keep_off, int32_t sum_keep,
+                      int32_t* keep_idx, float* q_tilde_out,
+                      void* ws, size_t ws_bytes, void* stream);
+
+/* Row compaction of the shortened sequence.  Output rows of image b, in
+ * order: system rows [0, S_b), visual rows S_b + keep_idx (ascending), text
+ * rows [S_b + N_V,b, T_b).  Output image b starts at row
+ * tok_off[b] - vis_off[b] + keep_off[b]; total rows sum_T - sum_vis + sum_keep.
+ *   src[i], dst[i]  n_tensors (1..32) HOST arrays of DEVICE pointers to
+ *                   row-major [sum_T][row] and [sum_T - sum_vis + sum_keep][row]
+ *                   tensors (e.g. hidden states and each layer's K and V).
+ *   row_bytes[i]    HOST array; each a positive multiple of 16; pointers
+ *                   16-byte aligned.
+ *   pos_ids_out     nullable int32 [total rows]: image-local original position
+ *                   of every output row.
+ * Requires 0 <= K_b <= N_V,b (device-checked; a violating image is skipped and
+ * E2S_ERR_SHAPE is raised in the status word).  Rows are copied bit-exactly. */
+e2s_status e2s_compact(const e2s_layout* layout, const int32_t* keep_idx,
+                       const int32_t* keep_off, int32_t sum_keep, int32_t n_tensors,
+                       const void* const* src, void* const* dst, const int64_t* row_bytes,
+                       int32_t* pos_ids_out, void* ws, size_t ws_bytes, void* stream);
+
+/* Synchronises `stream`, reads and returns the device status word (E2S_OK if
+ * no device-side error was recorded; otherwise the lowest-numbered recorded
+ * error).  Does not clear it. */
+e2s_status e2s_read_status(const void* ws, void* stream);
+
+/* Zeroes the device status word (stream-ordered, asynchronous). */
+e2s_status e2s_clear_status(void* ws, void* stream);
+
+/* Human-readable name of a status value (static string). */
+const char* e2s_status_string(e2s_status s);
+
+/* Library ABI version (major * 100 + minor). */
+int32_t e2s_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* E2S_H_ */

@@ -28,7 +28,8 @@ design notes as well):
     indices in ascending order.
   * Ablations (Table 2): NO_RELIABILITY rho = 1; NO_LAYER_FUSION uses the
     last layer only; NO_CONFLICT q = Pl; NO_NOVELTY lambda = 0; VANILLA ranks
-    by mean over layers and heads of a, with lambda = 0.
+    by mean over layers and heads of a, with lambda = 0.  NO_LAYER_FUSION
+    also ignores a carried prior (only the current layer's evidence).
 """
 from __future__ import annotations
 
@@ -325,7 +326,7 @@ def decide(q_text, k, n_sys, n_vis, n_text, grid_h, grid_w, keep, *, H_kv: int,
         a = image_scores(q_text, k, b, lay, H_kv, params.score_mode)
         ev = image_evidence(a, params)
         if params.flags & NO_LAYER_FUSION:
-            fused, K = fuse_layers(ev["mass"][-1:], None if prior is None else prior[v0:v1])
+            fused, K = fuse_layers(ev["mass"][-1:], None)
         else:
             fused, K = fuse_layers(ev["mass"], None if prior is None else prior[v0:v1])
         Pl = plausibility(fused)

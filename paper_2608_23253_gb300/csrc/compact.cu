@@ -1,0 +1,107 @@
+// Compaction of the retained rows: system rows, the kept visual rows and the
+// text rows of every image are gathered, in order, into the shortened
+// sequence that the next decoder layer consumes.  One warp per (tensor,
+// output row); 16-byte streaming loads and stores, fully coalesced.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+
+#include "device_common.cuh"
+
+namespace e2s {
+namespace {
+
+constexpr int kCompactThreads = 256;
+
+struct TensorSet {
+  const char* src[kMaxCompactTensors];
+  char* dst[kMaxCompactTensors];
+  int64_t row_bytes[kMaxCompactTensors];
+};
+
+// Largest b with out_off(b) <= r, out_off(b) = tok_off[b] - vis_off[b] + keep_off[b].
+__device__ __forceinline__ int out_image(const LayoutArgs& la, const int32_t* keep_off, int r) {
+  int lo = 0, hi = la.B - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    const int off = __ldg(la.tok_off + mid) - __ldg(la.vis_off + mid) + __ldg(keep_off + mid);
+    if (off <= r) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+__global__ void __launch_bounds__(kCompactThreads)
+    compact_kernel(const LayoutArgs la, const int32_t* __restrict__ keep_idx,
+                   const int32_t* __restrict__ keep_off, int n_tensors, const TensorSet ts,
+                   int32_t* __restrict__ pos_ids, long long total_rows, uint32_t* status) {
+  const int lane = threadIdx.x & 31;
+  const long long warps = (long long)gridDim.x * (blockDim.x >> 5);
+  const long long pairs = total_rows * n_tensors;
+  for (long long pr = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5; pr < pairs;
+       pr += warps) {
+    const int tix = (int)(pr / total_rows);
+    const int r = (int)(pr - (long long)tix * total_rows);
+    const int b = out_image(la, keep_off, r);
+    const int S = __ldg(la.n_sys + b), NV = __ldg(la.n_vis + b), NT = __ldg(la.n_text + b);
+    const int ko = __ldg(keep_off + b);
+    const int Kb = __ldg(keep_off + b + 1) - ko;
+    const int out0 = __ldg(la.tok_off + b) - __ldg(la.vis_off + b) + ko;
+    const int u = r - out0;
+    int src_local;
+    bool ok = Kb >= 0 && Kb <= NV && u >= 0 && u < S + Kb + NT;
+    if (u < S) {
+      src_local = u;
+    } else if (u < S + Kb) {
+      const int kv = __ldg(keep_idx + ko + (u - S));
+      ok = ok && kv >= 0 && kv < NV;
+      src_local = S + kv;
+    } else {
+      src_local = NV + u - Kb;
+    }
+    if (!ok) {
+      if (lane == 0) E2S_DEV_FLAG(status, E2S_ERR_SHAPE);
+      continue;
+    }
+    const long long src_row = (long long)__ldg(la.tok_off + b) + src_local;
+    const int64_t rb = ts.row_bytes[tix];
+    const uint4* s4 = reinterpret_cast<const uint4*>(ts.src[tix] + src_row * rb);
+    uint4* d4 = reinterpret_cast<uint4*>(ts.dst[tix] + (long long)r * rb);
+    const int n16 = (int)(rb >> 4);
+    int i = lane;
+    for (; i + 96 < n16; i += 128) {
+      const uint4 x0 = __ldcs(s4 + i), x1 = __ldcs(s4 + i + 32), x2 = __ldcs(s4 + i + 64),
+                  x3 = __ldcs(s4 + i + 96);
+      __stcs(d4 + i, x0);
+      __stcs(d4 + i + 32, x1);
+      __stcs(d4 + i + 64, x2);
+      __stcs(d4 + i + 96, x3);
+    }
+    for (; i < n16; i += 32) __stcs(d4 + i, __ldcs(s4 + i));
+    if (tix == 0 && lane == 0 && pos_ids) pos_ids[r] = src_local;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_compact(const LayoutArgs& la, const int32_t* keep_idx, const int32_t* keep_off,
+                           int32_t sum_keep, int32_t n_tensors, const void* const* src,
+                           void* const* dst, const int64_t* row_bytes, int32_t* pos_ids,
+                           uint32_t* status, cudaStream_t st) {
+  const long long total_rows = (long long)la.sum_T - la.sum_vis + sum_keep;
+  if (total_rows <= 0) return cudaSuccess;
+  TensorSet ts = {};
+  for (int i = 0; i < n_tensors; ++i) {
+    ts.src[i] = static_cast<const char*>(src[i]);
+    ts.dst[i] = static_cast<char*>(dst[i]);
+    ts.row_bytes[i] = row_bytes[i];
+  }
+  const long long pairs = total_rows * n_tensors;
+  const int warps_per_block = kCompactThreads / 32;
+  long long blocks = (pairs + warps_per_block - 1) / warps_per_block;
+  blocks = std::min<long long>(blocks, (long long)sm_count() * 16);
+  compact_kernel<<<(unsigned)std::max<long long>(blocks, 1), kCompactThreads, 0, st>>>(
+      la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status);
+  return cudaGetLastError();
+}
+
+}  // namespace e2s

@@ -1,0 +1,197 @@
+// C ABI of libe2s.so: argument validation and dispatch to the kernels.
+// Validation here is host-side only (sizes, pointers, alignment, enums);
+// the kernels re-check the device layout arrays and report through the
+// status word in the workspace.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "internal.h"
+
+namespace e2s {
+
+int sm_count() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 1;
+  return n > 0 ? n : 1;
+}
+
+namespace {
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+e2s_status check_layout(const e2s_layout* L) {
+  if (!L) return E2S_ERR_INVALID_ARG;
+  if (L->B < 1 || L->L < 1 || L->H < 1 || L->H_kv < 1) return E2S_ERR_SHAPE;
+  if (L->H % L->H_kv) return E2S_ERR_SHAPE;
+  if (L->d != 128) return E2S_ERR_UNSUPPORTED;
+  if (!L->tok_off || !L->n_sys || !L->n_vis || !L->n_text || !L->grid_h || !L->grid_w ||
+      !L->vis_off || !L->text_off)
+    return E2S_ERR_INVALID_ARG;
+  if (L->max_T < 0 || L->max_vis < 0 || L->max_text < 1 || L->sum_T < 0 || L->sum_vis < 0 ||
+      L->sum_text < L->B)
+    return E2S_ERR_SHAPE;
+  if (L->max_vis > L->max_T || L->max_text > L->max_T || L->sum_vis > L->sum_T ||
+      L->sum_text > L->sum_T || L->max_T > L->sum_T)
+    return E2S_ERR_SHAPE;
+  if (L->max_vis > 8192) return E2S_ERR_UNSUPPORTED;
+  if (L->max_text > 256) return E2S_ERR_UNSUPPORTED;
+  return E2S_OK;
+}
+
+e2s_status check_params(const e2s_params* P) {
+  if (!P) return E2S_ERR_INVALID_ARG;
+  if (P->score_mode != E2S_SCORE_EQ1 && P->score_mode != E2S_SCORE_CAUSAL_PROB)
+    return E2S_ERR_INVALID_ARG;
+  if (P->norm_mode < E2S_NORM_DEFAULT || P->norm_mode > E2S_NORM_RENORM) return E2S_ERR_INVALID_ARG;
+  if (P->score_mode == E2S_SCORE_EQ1 && P->norm_mode == E2S_NORM_RENORM) return E2S_ERR_UNSUPPORTED;
+  if (P->G < 1 || P->G > 8) return E2S_ERR_INVALID_ARG;
+  if (!(P->lambda >= 0.f && P->lambda <= 1.f)) return E2S_ERR_INVALID_ARG;
+  const uint32_t known = E2S_NO_RELIABILITY | E2S_NO_LAYER_FUSION | E2S_NO_CONFLICT |
+                         E2S_NO_NOVELTY | E2S_VANILLA | E2S_SIMT_SCORE;
+  if (P->flags & ~known) return E2S_ERR_INVALID_ARG;
+  return E2S_OK;
+}
+
+int norm_is_softmax(const e2s_params* P) {
+  if (P->norm_mode == E2S_NORM_SOFTMAX) return 1;
+  if (P->norm_mode == E2S_NORM_RENORM) return 0;
+  return P->score_mode == E2S_SCORE_EQ1 ? 1 : 0;
+}
+
+e2s_status check_ws(const e2s_layout* L, void* ws, size_t ws_bytes) {
+  if (!ws) return E2S_ERR_WORKSPACE;
+  if (reinterpret_cast<uintptr_t>(ws) & 255u) return E2S_ERR_WORKSPACE;
+  if (ws_bytes < kStatusBytes + stats_bytes(L)) return E2S_ERR_WORKSPACE;
+  return E2S_OK;
+}
+
+e2s_status from_cuda(cudaError_t e) { return e == cudaSuccess ? E2S_OK : E2S_ERR_CUDA; }
+
+#define E2S_TRY(x)                    \
+  do {                                \
+    const e2s_status s_ = (x);        \
+    if (s_ != E2S_OK) return s_;      \
+  } while (0)
+
+}  // namespace
+}  // namespace e2s
+
+using namespace e2s;
+
+extern "C" {
+
+size_t e2s_workspace_size(const e2s_layout* layout, const e2s_params* params) {
+  (void)params;
+  if (check_layout(layout) != E2S_OK) return 0;
+  return kStatusBytes + stats_bytes(layout);
+}
+
+e2s_status e2s_score(const e2s_layout* layout, const e2s_params* params, const void* q_text,
+                     int64_t q_row_stride, const void* k, int64_t k_row_stride, float* a_out,
+                     void* ws, size_t ws_bytes, void* stream) {
+  E2S_TRY(check_layout(layout));
+  E2S_TRY(check_params(params));
+  E2S_TRY(check_ws(layout, ws, ws_bytes));
+  if (!q_text || !k || (!a_out && layout->sum_vis > 0)) return E2S_ERR_INVALID_ARG;
+  if (q_row_stride < (int64_t)layout->H * layout->d || k_row_stride < (int64_t)layout->H_kv * layout->d)
+    return E2S_ERR_SHAPE;
+  if (!aligned16(q_text) || !aligned16(k) || (q_row_stride % 8) || (k_row_stride % 8))
+    return E2S_ERR_ALIGNMENT;
+  const LayoutArgs la = layout_args(layout);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (params->flags & E2S_SIMT_SCORE)
+    return from_cuda(launch_score_simt(la, params->score_mode, q_text, q_row_stride, k,
+                                       k_row_stride, a_out, status_word(ws), st));
+  int unsupported = 0;
+  const cudaError_t e = launch_score_tc(la, params->score_mode, q_text, q_row_stride, k,
+                                        k_row_stride, a_out, status_word(ws), st, &unsupported);
+  if (unsupported) return E2S_ERR_UNSUPPORTED;
+  return from_cuda(e);
+}
+
+e2s_status e2s_fuse(const e2s_layout* layout, const e2s_params* params, const float* a,
+                    const int32_t* cand, const float* prior, float* mass_out, float* fused_out,
+                    float* q_out, void* ws, size_t ws_bytes, void* stream) {
+  (void)cand;
+  E2S_TRY(check_layout(layout));
+  E2S_TRY(check_params(params));
+  E2S_TRY(check_ws(layout, ws, ws_bytes));
+  if (layout->sum_vis > 0 && (!a || !fused_out || !q_out)) return E2S_ERR_INVALID_ARG;
+  if (!aligned16(prior) || !aligned16(mass_out) || !aligned16(fused_out)) return E2S_ERR_ALIGNMENT;
+  return from_cuda(launch_fuse(layout_args(layout), norm_is_softmax(params), params->flags, a,
+                               prior, mass_out, fused_out, q_out, stats_ptr(ws), status_word(ws),
+                               static_cast<cudaStream_t>(stream)));
+}
+
+e2s_status e2s_select(const e2s_layout* layout, const e2s_params* params, const float* q,
+                      const int32_t* cand, const int32_t* keep_count, const int32_t* keep_off,
+                      int32_t sum_keep, int32_t* keep_idx, float* q_tilde_out, void* ws,
+                      size_t ws_bytes, void* stream) {
+  E2S_TRY(check_layout(layout));
+  E2S_TRY(check_params(params));
+  E2S_TRY(check_ws(layout, ws, ws_bytes));
+  if (!keep_count || !keep_off || sum_keep < 0) return E2S_ERR_INVALID_ARG;
+  if (layout->sum_vis > 0 && !q) return E2S_ERR_INVALID_ARG;
+  if (sum_keep > 0 && !keep_idx) return E2S_ERR_INVALID_ARG;
+  return from_cuda(launch_select(layout_args(layout), params->lambda, params->G, params->flags, q,
+                                 cand, keep_count, keep_off, sum_keep, keep_idx, q_tilde_out,
+                                 status_word(ws), static_cast<cudaStream_t>(stream)));
+}
+
+e2s_status e2s_compact(const e2s_layout* layout, const int32_t* keep_idx, const int32_t* keep_off,
+                       int32_t sum_keep, int32_t n_tensors, const void* const* src,
+                       void* const* dst, const int64_t* row_bytes, int32_t* pos_ids_out,
+                       void* ws, size_t ws_bytes, void* stream) {
+  E2S_TRY(check_layout(layout));
+  E2S_TRY(check_ws(layout, ws, ws_bytes));
+  if (!keep_off || sum_keep < 0 || sum_keep > layout->sum_vis) return E2S_ERR_SHAPE;
+  if (sum_keep > 0 && !keep_idx) return E2S_ERR_INVALID_ARG;
+  if (n_tensors < 0 || n_tensors > kMaxCompactTensors) return E2S_ERR_INVALID_ARG;
+  if (n_tensors > 0 && (!src || !dst || !row_bytes)) return E2S_ERR_INVALID_ARG;
+  for (int i = 0; i < n_tensors; ++i) {
+    if (!src[i] || !dst[i]) return E2S_ERR_INVALID_ARG;
+    if (row_bytes[i] <= 0) return E2S_ERR_SHAPE;
+    if ((row_bytes[i] & 15) || !aligned16(src[i]) || !aligned16(dst[i])) return E2S_ERR_ALIGNMENT;
+  }
+  if (n_tensors == 0 && !pos_ids_out) return E2S_OK;
+  return from_cuda(launch_compact(layout_args(layout), keep_idx, keep_off, sum_keep, n_tensors,
+                                  src, dst, row_bytes, pos_ids_out, status_word(ws),
+                                  static_cast<cudaStream_t>(stream)));
+}
+
+e2s_status e2s_read_status(const void* ws, void* stream) {
+  if (!ws) return E2S_ERR_WORKSPACE;
+  uint32_t word = 0;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&word, ws, sizeof(word), cudaMemcpyDeviceToHost, st) != cudaSuccess)
+    return E2S_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return E2S_ERR_CUDA;
+  for (int c = 1; c < 32; ++c)
+    if (word & (1u << c)) return static_cast<e2s_status>(c);
+  return E2S_OK;
+}
+
+e2s_status e2s_clear_status(void* ws, void* stream) {
+  if (!ws) return E2S_ERR_WORKSPACE;
+  return from_cuda(cudaMemsetAsync(ws, 0, sizeof(uint32_t), static_cast<cudaStream_t>(stream)));
+}
+
+const char* e2s_status_string(e2s_status s) {
+  switch (s) {
+    case E2S_OK: return "E2S_OK";
+    case E2S_ERR_INVALID_ARG: return "E2S_ERR_INVALID_ARG";
+    case E2S_ERR_SHAPE: return "E2S_ERR_SHAPE";
+    case E2S_ERR_ALIGNMENT: return "E2S_ERR_ALIGNMENT";
+    case E2S_ERR_UNSUPPORTED: return "E2S_ERR_UNSUPPORTED";
+    case E2S_ERR_WORKSPACE: return "E2S_ERR_WORKSPACE";
+    case E2S_ERR_CUDA: return "E2S_ERR_CUDA";
+    case E2S_ERR_TIMEOUT: return "E2S_ERR_TIMEOUT";
+  }
+  return "E2S_ERR_UNKNOWN";
+}
+
+int32_t e2s_version(void) { return 100; }
+
+}  // extern "C"
