@@ -140,6 +140,31 @@ e2s_status e2s_fuse(const e2s_layout* layout, const e2s_params* params,
                     float* mass_out, float* fused_out, float* q_out,
                     void* ws, size_t ws_bytes, void* stream);
 
+/* e2s_fuse without a workspace (the paper has no counterpart; this is a
+ * deployment convenience).  Some callers cannot allocate device memory: code
+ * running inside a host framework whose memory pool owns the whole device
+ * heap, plug-ins reached through a foreign-function interface that has no
+ * allocator, or real-time loops where cudaMalloc is not allowed.  This entry
+ * point takes the same inputs and outputs as e2s_fuse but keeps its scratch
+ * (the per-(image, layer, head) normalisation statistics) in a static device
+ * array inside the library, so it allocates nothing and needs no workspace.
+ *   - Capacity: B * L * H <= 8192; larger batches return E2S_ERR_WORKSPACE
+ *     before anything is launched.  The array (about 64 KiB) is held by every
+ *     GPU that loads the library until the process exits.
+ *   - The first call on a device looks up the array's device address (once
+ *     per device, with that device current); make that first call before any
+ *     stream capture.
+ *   - Every call shares the one array: calls whose kernels overlap on the GPU
+ *     (different streams, or different host threads on one device) race and
+ *     must be serialised by the caller.  Each call rewrites every statistic it
+ *     reads, so the contents left by an earlier call do no harm.
+ *   - Device-side layout errors are not reported (there is no status word to
+ *     read back); use e2s_fuse with a workspace and e2s_read_status to
+ *     diagnose them. */
+e2s_status e2s_fuse_noalloc(const e2s_layout* layout, const e2s_params* params,
+                            const float* a, const int32_t* cand, const float* prior,
+                            float* mass_out, float* fused_out, float* q_out, void* stream);
+
 /* Spatial novelty and Top-K (Sec. 4.3, Eqs. 20-23).
  *   q            fp32 [sum_vis] priorities (e2s_fuse q_out).
  *   cand         nullable int32 [sum_vis] original raster index of each slot

@@ -125,6 +125,22 @@ e2s_status e2s_fuse(const e2s_layout* layout, const e2s_params* params, const fl
                                static_cast<cudaStream_t>(stream)));
 }
 
+e2s_status e2s_fuse_noalloc(const e2s_layout* layout, const e2s_params* params, const float* a,
+                            const int32_t* cand, const float* prior, float* mass_out,
+                            float* fused_out, float* q_out, void* stream) {
+  (void)cand;
+  E2S_TRY(check_layout(layout));
+  E2S_TRY(check_params(params));
+  if (layout->sum_vis > 0 && (!a || !fused_out || !q_out)) return E2S_ERR_INVALID_ARG;
+  if (!aligned16(prior) || !aligned16(mass_out) || !aligned16(fused_out)) return E2S_ERR_ALIGNMENT;
+  int too_big = 0;
+  const cudaError_t e = launch_fuse_noalloc(layout_args(layout), norm_is_softmax(params),
+                                            params->flags, a, prior, mass_out, fused_out, q_out,
+                                            static_cast<cudaStream_t>(stream), &too_big);
+  if (too_big) return E2S_ERR_WORKSPACE;
+  return from_cuda(e);
+}
+
 e2s_status e2s_select(const e2s_layout* layout, const e2s_params* params, const float* q,
                       const int32_t* cand, const int32_t* keep_count, const int32_t* keep_off,
                       int32_t sum_keep, int32_t* keep_idx, float* q_tilde_out, void* ws,

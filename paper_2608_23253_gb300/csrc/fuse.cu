@@ -11,6 +11,8 @@
 //                      the token index.
 #include <cuda_runtime.h>
 
+#include <mutex>
+
 #include "device_common.cuh"
 
 namespace e2s {
@@ -150,6 +152,67 @@ cudaError_t launch_fuse(const LayoutArgs& la, int norm_softmax, uint32_t flags, 
       la, norm_softmax, flags, a, stats, reinterpret_cast<const float4*>(prior),
       reinterpret_cast<float4*>(mass_out), reinterpret_cast<float4*>(fused_out), q_out);
   return cudaGetLastError();
+}
+
+}  // namespace e2s
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant (e2s_fuse_noalloc).  Some callers cannot hand us a
+// workspace: code running inside a host framework whose memory pool owns the
+// device heap, plug-ins called through a foreign-function interface with no
+// allocator of their own, or real-time loops where any cudaMalloc is
+// forbidden.  For them the statistics scratch of e2s_fuse lives in this
+// file-scope device array instead.  Every GPU that loads the library holds it
+// until the process exits.
+namespace e2s {
+namespace {
+
+constexpr long long kNoAllocMaxUnits = 8192;   // images x layers x heads
+constexpr size_t kNoAllocBytes = kStatusBytes + (size_t)kNoAllocMaxUnits * sizeof(float2);
+static __device__ __align__(256) unsigned char g_fuse_scratch[kNoAllocBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_addr[kMaxDevices] = {};
+
+// Device address of g_fuse_scratch on the current device.  The host-side name
+// is only a stand-in, so the address is asked from the runtime once per
+// device (with that device current) and cached.
+cudaError_t scratch_address(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (g_scratch_addr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_fuse_scratch);
+    if (e != cudaSuccess) return e;
+    g_scratch_addr[dev] = p;
+  }
+  *out = g_scratch_addr[dev];
+  return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t launch_fuse_noalloc(const LayoutArgs& la, int norm_softmax, uint32_t flags,
+                                const float* a, const float* prior, float* mass_out,
+                                float* fused_out, float* q_out, cudaStream_t st, int* too_big) {
+  *too_big = 0;
+  if ((long long)la.B * la.L * la.H > kNoAllocMaxUnits) {
+    *too_big = 1;
+    return cudaSuccess;
+  }
+  void* base = nullptr;
+  const cudaError_t e = scratch_address(&base);
+  if (e != cudaSuccess) return e;
+  // The statistics are fully rewritten before they are read, so nothing left
+  // by an earlier call needs clearing; the status word is not read back.
+  uint32_t* status = static_cast<uint32_t*>(base);
+  float2* stats = reinterpret_cast<float2*>(static_cast<char*>(base) + kStatusBytes);
+  return launch_fuse(la, norm_softmax, flags, a, prior, mass_out, fused_out, q_out, stats, status,
+                     st);
 }
 
 }  // namespace e2s

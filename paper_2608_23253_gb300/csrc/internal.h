@@ -58,6 +58,11 @@ cudaError_t launch_score_simt(const LayoutArgs& la, int mode, const void* q, int
 cudaError_t launch_fuse(const LayoutArgs& la, int norm_softmax, uint32_t flags, const float* a,
                         const float* prior, float* mass_out, float* fused_out, float* q_out,
                         float2* stats, uint32_t* status, cudaStream_t st);
+// Same two kernels as launch_fuse, with the scratch in a static device array
+// (no workspace).  *too_big is set when B * L * H exceeds its capacity.
+cudaError_t launch_fuse_noalloc(const LayoutArgs& la, int norm_softmax, uint32_t flags,
+                                const float* a, const float* prior, float* mass_out,
+                                float* fused_out, float* q_out, cudaStream_t st, int* too_big);
 cudaError_t launch_select(const LayoutArgs& la, float lambda, int G, uint32_t flags,
                           const float* q, const int32_t* cand, const int32_t* keep_count,
                           const int32_t* keep_off, int32_t sum_keep, int32_t* keep_idx,

@@ -74,6 +74,7 @@ _SIGS = {
     "e2s_workspace_size": (_sz, [_LP, _PP]),
     "e2s_score": (ctypes.c_int, [_LP, _PP, _vp, _i64, _vp, _i64, _vp, _vp, _sz, _vp]),
     "e2s_fuse": (ctypes.c_int, [_LP, _PP, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "e2s_fuse_noalloc": (ctypes.c_int, [_LP, _PP, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
     "e2s_select": (ctypes.c_int, [_LP, _PP, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
     "e2s_compact": (ctypes.c_int, [_LP, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "e2s_read_status": (ctypes.c_int, [_vp, _vp]),
@@ -130,6 +131,13 @@ def e2s_fuse(layout, params_, a, cand, prior, mass_out, fused_out, q_out, ws, ws
     return lib.e2s_fuse(_ref(layout), _ref(params_), _ptr(a), _ptr(cand), _ptr(prior),
                         _ptr(mass_out), _ptr(fused_out), _ptr(q_out), _ptr(ws), ws_bytes,
                         _stream(stream))
+
+
+def e2s_fuse_noalloc(layout, params_, a, cand, prior, mass_out, fused_out, q_out,
+                     stream=None) -> int:
+    """e2s_fuse with its scratch in a static device array: no workspace, no allocation."""
+    return lib.e2s_fuse_noalloc(_ref(layout), _ref(params_), _ptr(a), _ptr(cand), _ptr(prior),
+                                _ptr(mass_out), _ptr(fused_out), _ptr(q_out), _stream(stream))
 
 
 def e2s_select(layout, params_, q, cand, keep_count, keep_off, sum_keep, keep_idx, q_tilde_out,
