@@ -33,9 +33,18 @@ import numpy as np  # noqa: E402
 
 METRIC = "pruning decisions/sec (images/s) at LLaVA-1.5 shape, K=64; % of HBM roofline"
 UNIT = "images/s"
-CFG_ID, KEEP = 1, 64
-WORKLOAD = "llava-1.5-7b decision+compaction, batch 1, 35+576(24x24)+64 tokens, 3 layers, " \
-           "32x128 MHA, K=64 (configs[1])"
+# name -> (config id, K, batch, description).  The default is the metric's
+# workload; the others exist for profiling and context lines.
+WORKLOADS = {
+    "cfg1": (1, 64, None, "llava-1.5-7b decision+compaction, batch 1, 35+576(24x24)+64 tokens, "
+                          "3 layers, 32x128 MHA, K=64 (configs[1])"),
+    "cfg2": (2, 64, None, "llava-1.5-7b decision+compaction, batch 32, 35+576(24x24)+U[16,128] "
+                          "ragged text tokens, 3 layers, 32x128 MHA, K=64 (configs[2])"),
+    "cfg3": (3, None, None, "qwen2-vl-7b decision+compaction, batch 16, grids 16x16..36x36, "
+                            "28q/4kv heads, 3 layers, K=11.1% (configs[3])"),
+    "cfg4": (4, None, None, "high-res decision+compaction, batch 8, 48x48/64x64 grids, 128 text, "
+                            "4 layers, 32x128 MHA, K=11% (configs[4])"),
+}
 
 # ncu dram__bytes_read.sum + dram__bytes_write.sum of one score-kernel launch on this
 # workload, and the sha256 (first 16 hex) of csrc/score_tc.cu when it was captured.
@@ -55,57 +64,84 @@ def measured_peaks():
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
-    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
-              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    """SM clocks and clock-event (throttle) reasons sampled through NVML every
+    ~2 ms on a background thread while the timed region runs (read-only
+    queries).  Falls back to nvidia-smi at 200 ms when NVML cannot be loaded."""
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
 
-    def __init__(self, index: int):
-        self.index = index
-        self.proc = None
-        self.lines = []
+    def __init__(self, uuid: str, index: int):
+        self.uuid, self.index = uuid, index
+        self.samples, self.reason_bits, self.max_mhz = [], 0, None
+        self._stop = threading.Event()
+        self._nvml = None
+        self._proc = None
+
+    def _open_nvml(self):
+        import ctypes
+        nv = ctypes.CDLL("libnvidia-ml.so.1")
+        if nv.nvmlInit_v2() != 0:
+            raise OSError("nvmlInit failed")
+        h = ctypes.c_void_p()
+        uuid = self.uuid if self.uuid.startswith("GPU-") else "GPU-" + self.uuid
+        if not hasattr(nv, "nvmlDeviceGetCurrentClocksEventReasons"):
+            raise OSError("NVML without clock-event reasons")
+        if nv.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(h)) != 0:
+            if nv.nvmlDeviceGetHandleByIndex_v2(self.index, ctypes.byref(h)) != 0:
+                raise OSError("no NVML handle")
+        mx = ctypes.c_uint()
+        if nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:
+            self.max_mhz = float(mx.value)
+        return nv, h
+
+    def _poll_nvml(self, nv, h):
+        import ctypes
+        clk, rs = ctypes.c_uint(), ctypes.c_ulonglong()
+        while not self._stop.is_set():
+            if nv.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0:
+                self.samples.append(float(clk.value))
+            if nv.nvmlDeviceGetCurrentClocksEventReasons(h, ctypes.byref(rs)) == 0:
+                self.reason_bits |= int(rs.value)
+            time.sleep(0.002)
+
+    def _poll_smi(self):
+        fields = "clocks.sm,clocks.max.sm,clocks_event_reasons.active"
+        self._proc = subprocess.Popen(
+            ["nvidia-smi", f"--id={self.index}", f"--query-gpu={fields}",
+             "--format=csv,noheader,nounits", "-lms", "200"],
+            stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        for line in self._proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            try:
+                self.samples.append(float(parts[0]))
+                self.max_mhz = float(parts[1])
+                self.reason_bits |= int(parts[2], 16)
+            except (ValueError, IndexError):
+                pass
 
     def __enter__(self):
         try:
-            self.proc = subprocess.Popen(
-                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
-                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
-            self.thread = threading.Thread(target=self._read, daemon=True)
-            self.thread.start()
+            nv, h = self._open_nvml()
+            target = lambda: self._poll_nvml(nv, h)  # noqa: E731
+            self.source = "nvml"
         except OSError:
-            self.proc = None
+            target = self._poll_smi
+            self.source = "nvidia-smi"
+        self._thread = threading.Thread(target=target, daemon=True)
+        self._thread.start()
         return self
 
-    def _read(self):
-        for line in self.proc.stdout:
-            self.lines.append(line.strip())
-
     def __exit__(self, *exc):
-        if self.proc is not None:
-            self.proc.terminate()
-            try:
-                self.proc.wait(timeout=5)
-            except subprocess.TimeoutExpired:
-                self.proc.kill()
+        self._stop.set()
+        if self._proc is not None:
+            self._proc.terminate()
+        self._thread.join(timeout=5)
 
     def summary(self):
-        sm, mx, reasons = [], None, set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
-            parts = [p.strip() for p in ln.split(",")]
-            if len(parts) < 8:
-                continue
-            try:
-                sm.append(float(parts[0]))
-                mx = float(parts[1])
-            except ValueError:
-                continue
-            for nm, val in zip(names, parts[4:8]):
-                if val.lower().startswith("active"):
-                    reasons.add(nm)
-        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
-                "reasons": sorted(reasons), "samples": len(sm)}
+        reasons = sorted(n for bit, n in self.REASONS.items() if self.reason_bits & bit)
+        return {"sm_mhz": statistics.median(self.samples) if self.samples else None,
+                "sm_max_mhz": self.max_mhz, "reasons": reasons, "samples": len(self.samples),
+                "source": self.source}
 
 
 def oracle_step(inp, params):
@@ -119,18 +155,18 @@ def oracle_step(inp, params):
     return ref
 
 
-def cpu_oracle_rate(seconds: float = 12.0, threads: int = 1):
+def cpu_oracle_rate(workload: str = "cfg1", seconds: float = 12.0, threads: int = 1):
     """Times the oracle (decision + compaction) on the host in a fresh process."""
     code = (
         "import sys,time,json;sys.path.insert(0,%r);import bench;"
         "from paper_2608_23253_gb300 import synth;"
         "from oracle import e2s_oracle as orc;"
-        "inp=synth.make_inputs(synth.config_spec(%d,keep=%d));p=orc.Params();"
+        "inp=synth.make_inputs(synth.config_spec(%d,keep=%r,batch=%r));p=orc.Params();"
         "bench.oracle_step(inp,p);n=0;t=time.perf_counter()\n"
         "while True:\n bench.oracle_step(inp,p);n+=1\n"
         " if time.perf_counter()-t>%f: break\n"
-        "print(json.dumps({'images':n,'seconds':time.perf_counter()-t}))"
-    ) % (ROOT, CFG_ID, KEEP, seconds)
+        "print(json.dumps({'images':n*inp.spec.B,'seconds':time.perf_counter()-t}))"
+    ) % (ROOT, WORKLOADS[workload][0], WORKLOADS[workload][1], WORKLOADS[workload][2], seconds)
     env = dict(os.environ)
     for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
         env[v] = str(threads)
@@ -154,15 +190,15 @@ def dist_setup(n_gpus: int):
 def run_reference(args, world, rank):
     if rank != 0:
         return
-    rate, info = cpu_oracle_rate(seconds=max(3.0, 3.0 * args.steps / 10.0 + 2.0))
+    rate, info = cpu_oracle_rate(args.workload, seconds=max(3.0, 3.0 * args.steps / 10.0 + 2.0))
     line = {
         "impl": "reference", "metric": METRIC, "value": rate, "unit": UNIT, "n_gpus": args.gpus,
         "steps": info["images"], "warmup": 1, "ms_per_step": 1e3 / rate,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": WORKLOAD},
+        "data": "synthetic", "config": {"workload": WORKLOADS[args.workload][3]},
         "cpu_baseline": {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
-                         "sample": f"{info['images']} decisions+compactions of one config-1 image "
-                                   f"in {info['seconds']:.1f} s, 1 thread"},
+                         "sample": f"decision+compaction of {info['images']} images of this "
+                                   f"workload in {info['seconds']:.1f} s, 1 thread"},
         "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -179,7 +215,8 @@ def run_ours(args, world, rank, local):
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
-    inp = synth.make_inputs(synth.config_spec(CFG_ID, keep=KEEP), with_payload=True)
+    cfg_id, keep, bsz, desc = WORKLOADS[args.workload]
+    inp = synth.make_inputs(synth.config_spec(cfg_id, keep=keep, batch=bsz), with_payload=True)
     s = inp.spec
     batch = Batch.from_inputs(inp, device=dev)
     dec = Decision(batch, inp.keep, e2s.params())
@@ -234,7 +271,7 @@ def run_ours(args, world, rank, local):
             torch.distributed.barrier()
         torch.cuda.synchronize()
         records = []
-        with ClockSampler(local) as clocks:
+        with ClockSampler(str(torch.cuda.get_device_properties(dev).uuid), local) as clocks:
             t_wall = time.perf_counter()
             for _ in range(args.steps):
                 evs = new_events()
@@ -309,9 +346,9 @@ def run_ours(args, world, rank, local):
         "warmup": args.warmup, "ms_per_step": statistics.mean(step_ms),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic",
-        "config": {"workload": WORKLOAD, "global_batch": batch.B * world, "seq_len": batch.sum_T,
+        "config": {"workload": desc, "global_batch": batch.B * world, "seq_len": batch.sum_T,
                    "n_vis": int(inp.n_vis[0]), "n_text": int(inp.n_text[0]), "layers": L,
-                   "keep": KEEP, "score_mode": "causal_prob", "norm": "renorm",
+                   "keep": int(inp.keep[0]), "score_mode": "causal_prob", "norm": "renorm",
                    "parallelism": f"replicas{world}",
                    "l2": "flushed before every step (256 MiB write)"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
@@ -329,10 +366,10 @@ def run_ours(args, world, rank, local):
         "wall_s_timed_region": t_wall,
     }
     if world == 1 and not args.no_cpu_baseline:
-        rate, info = cpu_oracle_rate()
+        rate, info = cpu_oracle_rate(args.workload)
         line["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
-                                "sample": f"{info['images']} decisions+compactions of one "
-                                          f"config-1 image in {info['seconds']:.1f} s, 1 thread"}
+                                "sample": f"decision+compaction of {info['images']} images of "
+                                          f"this workload in {info['seconds']:.1f} s, 1 thread"}
     print(json.dumps(line), flush=True)
 
 
@@ -343,6 +380,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="cfg1")
     args = ap.parse_args()
     if args.warmup < 3:
         raise SystemExit("--warmup must be >= 3")
