@@ -2,10 +2,14 @@
 
 One step = the whole hot path for one batch of the LLaVA-1.5-7B workload
 (35 system + 24x24 visual + 64 text tokens, 3 evidence layers, 32 heads x
-128, batch 1, K = 64): e2s_score (tcgen05, causal-prefix probability),
-e2s_fuse, e2s_select and e2s_compact of the hidden states and every evidence
-layer's K and V.  Inputs are seeded synthetic bf16 tensors (no dataset or
-checkpoint is available); L2 is flushed (256 MiB write) before every step.
+128, batch 1, K = 64): one e2s_prune call -- the tcgen05 score kernel
+(causal-prefix probability), the token-parallel evidence / fusion / Top-K
+kernel and the compaction of the hidden states and every evidence layer's K
+and V.  Inputs are seeded synthetic bf16 tensors (no dataset or checkpoint is
+available); L2 is flushed (256 MiB write) before every step.  The step is one
+CUDA graph (three kernels chained by programmatic dependent launch) between
+two event-record nodes; e2s_score, e2s_decide and e2s_compact are also
+replayed alone, each in its own graph, for the per-kernel times.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -233,59 +237,75 @@ def run_ours(args, world, rank, local):
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
 
     stream = torch.cuda.Stream(device=dev)
-    graphs = {}
+    import ctypes
+    cudart = ctypes.CDLL("libcudart.so.13")   # the runtime torch already loaded
+    cudart.cudaEventRecordWithFlags.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_uint]
+
+    def record_node(ev):
+        """Event record captured as a graph node (cudaEventRecordExternal)."""
+        rc = cudart.cudaEventRecordWithFlags(ctypes.c_void_p(ev.cuda_event),
+                                             ctypes.c_void_p(stream.cuda_stream), 1)
+        if rc != 0:
+            raise RuntimeError(f"cudaEventRecordWithFlags failed: {rc}")
+
+    step_call = lambda: dec.prune(q, k, src, dst, pos, stream=stream)   # noqa: E731
+    stages = ["score", "decide", "compact"]
+    calls = [lambda: dec.score(q, k, stream=stream),
+             lambda: dec.decide(q, k, stream=stream),
+             lambda: dec.compact(src, dst, pos, stream=stream)]
+
+    def capture(fns):
+        """One graph: event node, the calls (kernels chained by programmatic
+        dependent launch), event node."""
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        e1.record(stream)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            record_node(e0)
+            for fn in fns:
+                fn()
+            record_node(e1)
+        return g, e0, e1
+
     with torch.cuda.stream(stream):
-        # eager warm-up (also sets kernel attributes outside capture)
-        dec.score(q, k, stream=stream)
-        dec.fuse(stream=stream)
-        dec.select(stream=stream)
-        dec.compact(src, dst, pos, stream=stream)
+        for fn in calls + [step_call]:   # eager warm-up (sets kernel attributes outside capture)
+            fn()
         stream.synchronize()
         e2s.check(dec.status(stream), "device status after warm-up")
-        for name, fn in (("score", lambda: dec.score(q, k, stream=stream)),
-                         ("fuse_select", lambda: (dec.fuse(stream=stream),
-                                                  dec.select(stream=stream))),
-                         ("compact", lambda: dec.compact(src, dst, pos, stream=stream))):
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=stream):
-                fn()
-            graphs[name] = g
-    launches_per_step = 1 + 2 + 1 + 1
-    stages = list(graphs)
+        step_graph = capture([step_call])
+        stage_graphs = [capture([fn]) for fn in calls]
+    launches_per_step = 3   # score, evidence/fusion/Top-K, compaction
 
-    def step(evs):
+    def run(gx):
+        g, e0, e1 = gx
         flush.zero_()
-        evs[0].record(stream)
-        for i, name in enumerate(stages):
-            graphs[name].replay()
-            evs[i + 1].record(stream)
-
-    def new_events():
-        return [torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)]
+        g.replay()
+        stream.synchronize()
+        return e0.elapsed_time(e1)
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
-            step(new_events())
-        stream.synchronize()
+            run(step_graph)
         if world > 1:
             torch.distributed.barrier()
         torch.cuda.synchronize()
-        records = []
         with ClockSampler(str(torch.cuda.get_device_properties(dev).uuid), local) as clocks:
             t_wall = time.perf_counter()
-            for _ in range(args.steps):
-                evs = new_events()
-                step(evs)
-                records.append(evs)
-            stream.synchronize()
+            step_ms = [run(step_graph) for _ in range(args.steps)]
             torch.cuda.synchronize()
             t_wall = time.perf_counter() - t_wall
+            # each stage alone (same inputs, L2 flushed before every replay): the
+            # per-kernel durations behind the roofline fractions
+            n_stage = max(args.steps // 4, 10)
+            for gx in stage_graphs:
+                for _ in range(3):
+                    run(gx)
+            stage_ms = {name: [run(gx) for _ in range(n_stage)]
+                        for name, gx in zip(stages, stage_graphs)}
         if world > 1:
             torch.distributed.barrier()
         e2s.check(dec.status(stream), "device status after timing")
-        stage_ms = {name: [ev[i].elapsed_time(ev[i + 1]) for ev in records]
-                    for i, name in enumerate(stages)}
-        step_ms = [ev[0].elapsed_time(ev[-1]) for ev in records]
 
         # end to end through the public API, host buffers in pinned memory
         host_in = [torch.from_numpy(x.view(np.int16)).pin_memory()
@@ -301,8 +321,7 @@ def run_ours(args, world, rank, local):
             e0.record(stream)
             for hsrc, ddst in zip(host_in, dev_in):
                 ddst.view(torch.int16).view(-1).copy_(hsrc.view(-1), non_blocking=True)
-            for name in stages:
-                graphs[name].replay()
+            step_graph[0].replay()
             out_keep.copy_(dec.keep_idx, non_blocking=True)
             out_pos.copy_(pos, non_blocking=True)
             e1.record(stream)
@@ -320,16 +339,22 @@ def run_ours(args, world, rank, local):
     images = batch.B * args.steps * world
     value = images / (total_ms * 1e-3)
 
-    # roofline of the dominant kernel
+    # roofline of the dominant kernel.  Algorithmic bytes: score reads K of the
+    # whole sequence and the text queries once and writes a; the decision
+    # kernel reads a and the statistics and writes masses, fused mass, q, q~
+    # and the keep lists; the compaction reads and writes every retained row.
     L, H, Hkv, d = s.L, s.H, s.H_kv, s.d
     bytes_stage = {
         "score": L * batch.sum_T * Hkv * d * 2 + L * batch.sum_text * H * d * 2
                  + L * H * batch.sum_vis * 4,
-        "fuse_select": L * H * batch.sum_vis * 4 * 3 + L * batch.sum_vis * 16
-                       + batch.sum_vis * (16 + 4 + 4) + dec.sum_keep * 4,
+        "decide": L * H * batch.sum_vis * 4 + batch.B * L * H * 16 + L * batch.sum_vis * 16
+                  + batch.sum_vis * (16 + 4 + 4) + dec.sum_keep * 4,
         "compact": 2 * R * sum(t.stride(0) * t.element_size() for t in src) + R * 4,
     }
     mean_ms = {n: statistics.mean(v_) for n, v_ in stage_ms.items()}
+    # e2s_decide is the score kernel plus the decision kernel: the decision
+    # kernel's own time is the difference of the two isolated graphs
+    mean_ms["decide"] = max(mean_ms["decide"] - mean_ms["score"], 1e-6)
     dom = max(mean_ms, key=mean_ms.get)
     peaks = measured_peaks()
     peak, peak_src = (peaks["hbm_gbs"], "measured") if peaks else (6800.0, "fallback")
@@ -355,6 +380,8 @@ def run_ours(args, world, rank, local):
                      "frac": achieved / peak, "traffic": traffic, "kernel": dom,
                      "peak_source": f"{peak_src} hbm_gbs",
                      "algorithmic_bytes": bytes_stage[dom]},
+        "stages_note": "each stage replayed alone, L2 flushed; decide = e2s_decide graph "
+                       "minus e2s_score graph (the decision kernel's incremental time)",
         "stages": {n: {"us": mean_ms[n] * 1e3, "algorithmic_bytes": bytes_stage[n],
                        "GB/s": bytes_stage[n] / (mean_ms[n] * 1e-3) / 1e9,
                        "frac_hbm": bytes_stage[n] / (mean_ms[n] * 1e-3) / 1e9 / peak}

@@ -102,9 +102,11 @@ typedef struct {
   uint32_t flags;      /* E2S_* flags                                            */
 } e2s_params;
 
-/* Bytes of workspace every call below needs (status word + per-(image, layer,
- * head) normalisation statistics).  The workspace must be 256-byte aligned
- * and its first 4 bytes zero before the first call (see e2s_clear_status). */
+/* Bytes of workspace every call below needs: the status word, one float4 of
+ * normalisation statistics per (image, layer, head) written by e2s_score and
+ * e2s_decide, and one arrival counter per image (e2s_decide).  The workspace
+ * must be 256-byte aligned and its first 4 bytes zero before the first call
+ * (see e2s_clear_status); the rest needs no initialisation. */
 size_t e2s_workspace_size(const e2s_layout* layout, const e2s_params* params);
 
 /* Text-to-visual score (Sec. 3.1, Eq. 1; Algorithm 1 "Compute a_{l,h,n}").
@@ -122,11 +124,53 @@ e2s_status e2s_score(const e2s_layout* layout, const e2s_params* params,
                      const void* k, int64_t k_row_stride,
                      float* a_out, void* ws, size_t ws_bytes, void* stream);
 
+/* The whole pruning decision of one step in two launches: e2s_score, then
+ * evidence, fusion and selection (Sec. 3.1 and 4.1-4.3, Eqs. 1 and 8-23).
+ * Arguments have the meaning they have in e2s_score, e2s_fuse and e2s_select;
+ * a_out is required (it carries a[l][h][n] from the first launch to the
+ * second).  The score kernel also leaves the Eq. 8 normalisation statistics
+ * of every (image, layer, head) in the workspace, so the second kernel treats
+ * every visual token independently (64 tokens per CTA) and the last CTA to
+ * finish an image runs that image's Top-K.  Results are identical to
+ * e2s_score, e2s_fuse and e2s_select called in sequence, up to the rounding
+ * order of the normalisation sums.  keep_count and keep_off are required;
+ * keep_idx may be NULL only when sum_keep == 0.  Concurrent e2s_decide calls
+ * must use separate workspaces.  E2S_ERR_UNSUPPORTED when H > 384 or
+ * L * H > 4096. */
+e2s_status e2s_decide(const e2s_layout* layout, const e2s_params* params,
+                      const void* q_text, int64_t q_row_stride,
+                      const void* k, int64_t k_row_stride,
+                      const int32_t* cand, const float* prior, float* a_out,
+                      float* mass_out, float* fused_out, float* q_out,
+                      const int32_t* keep_count, const int32_t* keep_off, int32_t sum_keep,
+                      int32_t* keep_idx, float* q_tilde_out,
+                      void* ws, size_t ws_bytes, void* stream);
+
+/* One complete pruning step: e2s_decide followed by e2s_compact, three
+ * launches (Algorithm 1, one pruning layer; Sec. 3.1 and 4.1-4.3).  Arguments
+ * are those of the two calls.  Because the score kernel starts only after all
+ * earlier work on the stream, the compaction copies the system and text rows
+ * (which do not depend on the selection) while the decision is still running
+ * and waits only before the kept visual rows.  The src tensors, keep_count
+ * and keep_off must therefore be written by earlier work on the same stream
+ * (or be complete before the call), and nothing else may write them while
+ * the call runs.  Results are identical to e2s_decide then e2s_compact. */
+e2s_status e2s_prune(const e2s_layout* layout, const e2s_params* params,
+                     const void* q_text, int64_t q_row_stride,
+                     const void* k, int64_t k_row_stride,
+                     const int32_t* cand, const float* prior, float* a_out,
+                     float* mass_out, float* fused_out, float* q_out,
+                     const int32_t* keep_count, const int32_t* keep_off, int32_t sum_keep,
+                     int32_t* keep_idx, float* q_tilde_out,
+                     int32_t n_tensors, const void* const* src, void* const* dst,
+                     const int64_t* row_bytes, int32_t* pos_ids_out,
+                     void* ws, size_t ws_bytes, void* stream);
+
 /* Evidence and fusion (Sec. 4.1-4.2, Eqs. 8-19; Algorithm 1 inner loops).
  *   a          fp32 [L][H][sum_vis] from e2s_score.
  *   cand       nullable int32 [sum_vis]: original raster index of visual slot n
- *              (a later progressive step); NULL = identity.  Only e2s_select
- *              reads it; accepted here for symmetry and ignored.
+ *              (a later progressive step); NULL = identity.  Only the spatial
+ *              cells of the Top-K read it; e2s_fuse accepts it for symmetry.
  *   prior      nullable fp32 [sum_vis][4] (m~(I), m~(U), m~(Theta), -): fused
  *              mass carried from an earlier pruning step.  NULL: the first
  *              layer initialises the fusion (Eq. 12) and K^(1) = 0.
@@ -140,14 +184,26 @@ e2s_status e2s_fuse(const e2s_layout* layout, const e2s_params* params,
                     float* mass_out, float* fused_out, float* q_out,
                     void* ws, size_t ws_bytes, void* stream);
 
+/* e2s_fuse followed by e2s_select in a single launch (one thread-block cluster
+ * per image; Sec. 4.1-4.3, Eqs. 8-23).  Arguments and outputs are those of the
+ * two calls; results are identical to calling them in sequence. */
+e2s_status e2s_fuse_select(const e2s_layout* layout, const e2s_params* params,
+                           const float* a, const int32_t* cand, const float* prior,
+                           float* mass_out, float* fused_out, float* q_out,
+                           const int32_t* keep_count, const int32_t* keep_off, int32_t sum_keep,
+                           int32_t* keep_idx, float* q_tilde_out,
+                           void* ws, size_t ws_bytes, void* stream);
+
 /* e2s_fuse without a workspace (the paper has no counterpart; this is a
  * deployment convenience).  Some callers cannot allocate device memory: code
  * running inside a host framework whose memory pool owns the whole device
  * heap, plug-ins reached through a foreign-function interface that has no
  * allocator, or real-time loops where cudaMalloc is not allowed.  This entry
- * point takes the same inputs and outputs as e2s_fuse but keeps its scratch
- * (the per-(image, layer, head) normalisation statistics) in a static device
- * array inside the library, so it allocates nothing and needs no workspace.
+ * point takes the same inputs and outputs as e2s_fuse and computes the same
+ * results with a two-kernel formulation (a statistics kernel, then one thread
+ * per token) whose scratch -- the per-(image, layer, head) normalisation
+ * statistics -- lives in a static device array inside the library, so it
+ * allocates nothing and needs no workspace.
  *   - Capacity: B * L * H <= 8192; larger batches return E2S_ERR_WORKSPACE
  *     before anything is launched.  The array (about 64 KiB) is held by every
  *     GPU that loads the library until the process exits.

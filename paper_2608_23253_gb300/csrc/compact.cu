@@ -12,6 +12,7 @@ namespace e2s {
 namespace {
 
 constexpr int kCompactThreads = 256;
+constexpr int kRowVec = 16;   // 16-byte vectors per lane in flight
 
 struct TensorSet {
   const char* src[kMaxCompactTensors];
@@ -30,13 +31,17 @@ __device__ __forceinline__ int out_image(const LayoutArgs& la, const int32_t* ke
   return lo;
 }
 
-__global__ void __launch_bounds__(kCompactThreads)
-    compact_kernel(const LayoutArgs la, const int32_t* __restrict__ keep_idx,
-                   const int32_t* __restrict__ keep_off, int n_tensors, const TensorSet ts,
-                   int32_t* __restrict__ pos_ids, long long total_rows, uint32_t* status) {
+// One (tensor, output row) pair per warp, grid-stride.  visual < 0: every
+// row; visual == 0: system and text rows only; visual == 1: kept visual rows
+// only.
+__device__ __forceinline__ void compact_rows(const LayoutArgs& la, const int32_t* keep_idx,
+                                             const int32_t* keep_off, int n_tensors,
+                                             const TensorSet& ts, int32_t* pos_ids,
+                                             long long total_rows, uint32_t* status, int visual) {
   const int lane = threadIdx.x & 31;
   const long long warps = (long long)gridDim.x * (blockDim.x >> 5);
-  const long long pairs = total_rows * n_tensors;
+  // with no tensors the pass still writes the position ids
+  const long long pairs = total_rows * (n_tensors > 0 ? n_tensors : 1);
   for (long long pr = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5; pr < pairs;
        pr += warps) {
     const int tix = (int)(pr / total_rows);
@@ -47,11 +52,13 @@ __global__ void __launch_bounds__(kCompactThreads)
     const int Kb = __ldg(keep_off + b + 1) - ko;
     const int out0 = __ldg(la.tok_off + b) - __ldg(la.vis_off + b) + ko;
     const int u = r - out0;
+    const bool is_vis = u >= S && u < S + Kb;
+    if (visual >= 0 && is_vis != (visual == 1)) continue;
     int src_local;
     bool ok = Kb >= 0 && Kb <= NV && u >= 0 && u < S + Kb + NT;
     if (u < S) {
       src_local = u;
-    } else if (u < S + Kb) {
+    } else if (is_vis) {
       const int kv = __ldg(keep_idx + ko + (u - S));
       ok = ok && kv >= 0 && kv < NV;
       src_local = S + kv;
@@ -62,22 +69,47 @@ __global__ void __launch_bounds__(kCompactThreads)
       if (lane == 0) E2S_DEV_FLAG(status, E2S_ERR_SHAPE);
       continue;
     }
+    if (tix == 0 && lane == 0 && pos_ids) pos_ids[r] = src_local;
+    if (n_tensors == 0) continue;
     const long long src_row = (long long)__ldg(la.tok_off + b) + src_local;
     const int64_t rb = ts.row_bytes[tix];
     const uint4* s4 = reinterpret_cast<const uint4*>(ts.src[tix] + src_row * rb);
     uint4* d4 = reinterpret_cast<uint4*>(ts.dst[tix] + (long long)r * rb);
     const int n16 = (int)(rb >> 4);
-    int i = lane;
-    for (; i + 96 < n16; i += 128) {
-      const uint4 x0 = __ldcs(s4 + i), x1 = __ldcs(s4 + i + 32), x2 = __ldcs(s4 + i + 64),
-                  x3 = __ldcs(s4 + i + 96);
-      __stcs(d4 + i, x0);
-      __stcs(d4 + i + 32, x1);
-      __stcs(d4 + i + 64, x2);
-      __stcs(d4 + i + 96, x3);
+    // up to 8 KiB of the row in flight per warp: all loads first, then stores
+    for (int base = 0; base < n16; base += 32 * kRowVec) {
+      uint4 x[kRowVec];
+#pragma unroll
+      for (int v = 0; v < kRowVec; ++v) {
+        const int i = base + v * 32 + lane;
+        if (i < n16) x[v] = __ldcs(s4 + i);
+      }
+#pragma unroll
+      for (int v = 0; v < kRowVec; ++v) {
+        const int i = base + v * 32 + lane;
+        if (i < n16) __stcs(d4 + i, x[v]);
+      }
     }
-    for (; i < n16; i += 32) __stcs(d4 + i, __ldcs(s4 + i));
-    if (tix == 0 && lane == 0 && pos_ids) pos_ids[r] = src_local;
+  }
+}
+
+// early != 0: the system and text rows (which do not depend on the selection)
+// are copied before griddepcontrol.wait, overlapping the kernel that writes
+// keep_idx; the caller guarantees that the sources and keep_off were complete
+// before that kernel's predecessor started.
+__global__ void __launch_bounds__(kCompactThreads)
+    compact_kernel(const LayoutArgs la, const int32_t* __restrict__ keep_idx,
+                   const int32_t* __restrict__ keep_off, int n_tensors, const TensorSet ts,
+                   int32_t* __restrict__ pos_ids, long long total_rows, uint32_t* status,
+                   int early) {
+  pdl_launch_dependents();
+  if (early) {
+    compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, 0);
+    pdl_wait();   // keep_idx comes from the previous kernel
+    compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, 1);
+  } else {
+    pdl_wait();
+    compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, -1);
   }
 }
 
@@ -86,7 +118,7 @@ __global__ void __launch_bounds__(kCompactThreads)
 cudaError_t launch_compact(const LayoutArgs& la, const int32_t* keep_idx, const int32_t* keep_off,
                            int32_t sum_keep, int32_t n_tensors, const void* const* src,
                            void* const* dst, const int64_t* row_bytes, int32_t* pos_ids,
-                           uint32_t* status, cudaStream_t st) {
+                           uint32_t* status, cudaStream_t st, int early) {
   const long long total_rows = (long long)la.sum_T - la.sum_vis + sum_keep;
   if (total_rows <= 0) return cudaSuccess;
   TensorSet ts = {};
@@ -95,13 +127,13 @@ cudaError_t launch_compact(const LayoutArgs& la, const int32_t* keep_idx, const 
     ts.dst[i] = static_cast<char*>(dst[i]);
     ts.row_bytes[i] = row_bytes[i];
   }
-  const long long pairs = total_rows * n_tensors;
+  const long long pairs = total_rows * (n_tensors > 0 ? n_tensors : 1);
   const int warps_per_block = kCompactThreads / 32;
   long long blocks = (pairs + warps_per_block - 1) / warps_per_block;
   blocks = std::min<long long>(blocks, (long long)sm_count() * 16);
-  compact_kernel<<<(unsigned)std::max<long long>(blocks, 1), kCompactThreads, 0, st>>>(
-      la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status);
-  return cudaGetLastError();
+  return launch_kernel(compact_kernel, dim3((unsigned)std::max<long long>(blocks, 1)),
+                       dim3(kCompactThreads), 0, st, 0, true, la, keep_idx, keep_off, n_tensors, ts,
+                       pos_ids, total_rows, status, early);
 }
 
 }  // namespace e2s

@@ -13,11 +13,24 @@ constexpr float kNegBig = -1.0e30f;   // finite "minus infinity" for (max, sum) 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
+// Hardware base-2 exponential (MUFU ex2, flush-to-zero; max relative error
+// about 2^-22) and reciprocal.
+__device__ __forceinline__ float fast_ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float fast_rcp(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // Merge two online-softmax partials (m, l) in the log2 domain:
 // l * 2^m + l2 * 2^m2 = l' * 2^max(m, m2).  One exp2 per merge.
 __device__ __forceinline__ void lse_merge(float& m, float& l, float m2, float l2) {
   const float mx = fmaxf(m, m2);
-  const float e = exp2f(fminf(m, m2) - mx);
+  const float e = fast_ex2(fminf(m, m2) - mx);
   l = (m >= m2) ? fmaf(l2, e, l) : fmaf(l, e, l2);
   m = mx;
 }
@@ -28,11 +41,26 @@ __device__ __forceinline__ uint32_t ordered_key(float x) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
+// Workspace entry of the Eq. 8 normalisation statistics of one (image, layer,
+// head) row of visual scores, from S = sum a, M = max a*log2e and
+// E = sum 2^(a*log2e - M): (S, M, 1/E, 1/S), a reciprocal 0 when its sum is not
+// positive.
+__device__ __forceinline__ float4 stats_entry(float S, float M, float E) {
+  return make_float4(S, M, E > 0.f ? 1.f / E : 0.f, S > 0.f ? 1.f / S : 0.f);
+}
+
 __device__ __forceinline__ uint64_t globaltimer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
+
+// Programmatic dependent launch: let the next kernel on the stream be
+// scheduled now / wait until the previous kernel's writes are visible.
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 // Block-wide reductions for blockDim.x a multiple of 32 (<= 1024).
 template <typename F>

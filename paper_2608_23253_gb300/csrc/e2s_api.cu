@@ -63,7 +63,7 @@ int norm_is_softmax(const e2s_params* P) {
 e2s_status check_ws(const e2s_layout* L, void* ws, size_t ws_bytes) {
   if (!ws) return E2S_ERR_WORKSPACE;
   if (reinterpret_cast<uintptr_t>(ws) & 255u) return E2S_ERR_WORKSPACE;
-  if (ws_bytes < kStatusBytes + stats_bytes(L)) return E2S_ERR_WORKSPACE;
+  if (ws_bytes < kStatusBytes + stats_bytes(L) + decide_scratch_bytes(L)) return E2S_ERR_WORKSPACE;
   return E2S_OK;
 }
 
@@ -75,6 +75,89 @@ e2s_status from_cuda(cudaError_t e) { return e == cudaSuccess ? E2S_OK : E2S_ERR
     if (s_ != E2S_OK) return s_;      \
   } while (0)
 
+e2s_status check_score_args(const e2s_layout* layout, const void* q_text, int64_t q_row_stride,
+                            const void* k, int64_t k_row_stride, const float* a_out) {
+  if (!q_text || !k || (!a_out && layout->sum_vis > 0)) return E2S_ERR_INVALID_ARG;
+  if (q_row_stride < (int64_t)layout->H * layout->d ||
+      k_row_stride < (int64_t)layout->H_kv * layout->d)
+    return E2S_ERR_SHAPE;
+  if (!aligned16(q_text) || !aligned16(k) || (q_row_stride % 8) || (k_row_stride % 8))
+    return E2S_ERR_ALIGNMENT;
+  return E2S_OK;
+}
+
+// Score launch shared by e2s_score and e2s_decide; the decision scratch it
+// zeroes may be null.
+e2s_status run_score(const e2s_layout* layout, const e2s_params* params, const void* q_text,
+                     int64_t q_row_stride, const void* k, int64_t k_row_stride, float* a_out,
+                     void* ws, uint32_t* counters, cudaStream_t st) {
+  const LayoutArgs la = layout_args(layout);
+  if (params->flags & E2S_SIMT_SCORE)
+    return from_cuda(launch_score_simt(la, params->score_mode, q_text, q_row_stride, k,
+                                       k_row_stride, a_out, stats_ptr(ws), counters,
+                                       status_word(ws), st));
+  int unsupported = 0;
+  const cudaError_t e =
+      launch_score_tc(la, params->score_mode, q_text, q_row_stride, k, k_row_stride, a_out,
+                      stats_ptr(ws), counters, status_word(ws), st, &unsupported);
+  if (unsupported) return E2S_ERR_UNSUPPORTED;
+  return from_cuda(e);
+}
+
+e2s_status check_decide_args(const e2s_layout* layout, const e2s_params* params,
+                             const void* q_text, int64_t q_row_stride, const void* k,
+                             int64_t k_row_stride, const float* prior, const float* a_out,
+                             const float* mass_out, const float* fused_out, const float* q_out,
+                             const int32_t* keep_count, const int32_t* keep_off, int32_t sum_keep,
+                             const int32_t* keep_idx, void* ws, size_t ws_bytes) {
+  E2S_TRY(check_layout(layout));
+  E2S_TRY(check_params(params));
+  E2S_TRY(check_ws(layout, ws, ws_bytes));
+  E2S_TRY(check_score_args(layout, q_text, q_row_stride, k, k_row_stride, a_out));
+  if (layout->sum_vis > 0 && (!fused_out || !q_out)) return E2S_ERR_INVALID_ARG;
+  if (!keep_count || !keep_off || sum_keep < 0) return E2S_ERR_INVALID_ARG;
+  if (sum_keep > 0 && !keep_idx) return E2S_ERR_INVALID_ARG;
+  if (!aligned16(prior) || !aligned16(mass_out) || !aligned16(fused_out)) return E2S_ERR_ALIGNMENT;
+  if (!decide_fits(layout_args(layout))) return E2S_ERR_UNSUPPORTED;
+  return E2S_OK;
+}
+
+// Score (zeroing the arrival counters), then the token-parallel decision.
+e2s_status run_decide(const e2s_layout* layout, const e2s_params* params, const void* q_text,
+                      int64_t q_row_stride, const void* k, int64_t k_row_stride,
+                      const int32_t* cand, const float* prior, float* a_out, float* mass_out,
+                      float* fused_out, float* q_out, const int32_t* keep_count,
+                      const int32_t* keep_off, int32_t sum_keep, int32_t* keep_idx,
+                      float* q_tilde_out, void* ws, cudaStream_t st) {
+  uint32_t* scratch = decide_scratch_ptr(ws, layout);
+  E2S_TRY(run_score(layout, params, q_text, q_row_stride, k, k_row_stride, a_out, ws, scratch,
+                    st));
+  int unsupported = 0;
+  const cudaError_t e =
+      launch_decide(layout_args(layout), norm_is_softmax(params), params->flags, params->lambda,
+                    params->G, a_out, stats_ptr(ws), prior, cand, mass_out, fused_out, q_out,
+                    q_tilde_out, keep_count, keep_off, sum_keep, keep_idx, scratch,
+                    status_word(ws), st, &unsupported);
+  if (unsupported) return E2S_ERR_UNSUPPORTED;
+  return from_cuda(e);
+}
+
+e2s_status check_compact_args(const e2s_layout* layout, const int32_t* keep_idx,
+                              const int32_t* keep_off, int32_t sum_keep, int32_t n_tensors,
+                              const void* const* src, void* const* dst,
+                              const int64_t* row_bytes) {
+  if (!keep_off || sum_keep < 0 || sum_keep > layout->sum_vis) return E2S_ERR_SHAPE;
+  if (sum_keep > 0 && !keep_idx) return E2S_ERR_INVALID_ARG;
+  if (n_tensors < 0 || n_tensors > kMaxCompactTensors) return E2S_ERR_INVALID_ARG;
+  if (n_tensors > 0 && (!src || !dst || !row_bytes)) return E2S_ERR_INVALID_ARG;
+  for (int i = 0; i < n_tensors; ++i) {
+    if (!src[i] || !dst[i]) return E2S_ERR_INVALID_ARG;
+    if (row_bytes[i] <= 0) return E2S_ERR_SHAPE;
+    if ((row_bytes[i] & 15) || !aligned16(src[i]) || !aligned16(dst[i])) return E2S_ERR_ALIGNMENT;
+  }
+  return E2S_OK;
+}
+
 }  // namespace
 }  // namespace e2s
 
@@ -85,7 +168,7 @@ extern "C" {
 size_t e2s_workspace_size(const e2s_layout* layout, const e2s_params* params) {
   (void)params;
   if (check_layout(layout) != E2S_OK) return 0;
-  return kStatusBytes + stats_bytes(layout);
+  return kStatusBytes + stats_bytes(layout) + decide_scratch_bytes(layout);
 }
 
 e2s_status e2s_score(const e2s_layout* layout, const e2s_params* params, const void* q_text,
@@ -94,35 +177,87 @@ e2s_status e2s_score(const e2s_layout* layout, const e2s_params* params, const v
   E2S_TRY(check_layout(layout));
   E2S_TRY(check_params(params));
   E2S_TRY(check_ws(layout, ws, ws_bytes));
-  if (!q_text || !k || (!a_out && layout->sum_vis > 0)) return E2S_ERR_INVALID_ARG;
-  if (q_row_stride < (int64_t)layout->H * layout->d || k_row_stride < (int64_t)layout->H_kv * layout->d)
-    return E2S_ERR_SHAPE;
-  if (!aligned16(q_text) || !aligned16(k) || (q_row_stride % 8) || (k_row_stride % 8))
-    return E2S_ERR_ALIGNMENT;
-  const LayoutArgs la = layout_args(layout);
+  E2S_TRY(check_score_args(layout, q_text, q_row_stride, k, k_row_stride, a_out));
+  return run_score(layout, params, q_text, q_row_stride, k, k_row_stride, a_out, ws, nullptr,
+                   static_cast<cudaStream_t>(stream));
+}
+
+e2s_status e2s_decide(const e2s_layout* layout, const e2s_params* params, const void* q_text,
+                      int64_t q_row_stride, const void* k, int64_t k_row_stride,
+                      const int32_t* cand, const float* prior, float* a_out, float* mass_out,
+                      float* fused_out, float* q_out, const int32_t* keep_count,
+                      const int32_t* keep_off, int32_t sum_keep, int32_t* keep_idx,
+                      float* q_tilde_out, void* ws, size_t ws_bytes, void* stream) {
+  E2S_TRY(check_decide_args(layout, params, q_text, q_row_stride, k, k_row_stride, prior, a_out,
+                            mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
+                            ws, ws_bytes));
+  return run_decide(layout, params, q_text, q_row_stride, k, k_row_stride, cand, prior, a_out,
+                    mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
+                    q_tilde_out, ws, static_cast<cudaStream_t>(stream));
+}
+
+e2s_status e2s_prune(const e2s_layout* layout, const e2s_params* params, const void* q_text,
+                     int64_t q_row_stride, const void* k, int64_t k_row_stride,
+                     const int32_t* cand, const float* prior, float* a_out, float* mass_out,
+                     float* fused_out, float* q_out, const int32_t* keep_count,
+                     const int32_t* keep_off, int32_t sum_keep, int32_t* keep_idx,
+                     float* q_tilde_out, int32_t n_tensors, const void* const* src,
+                     void* const* dst, const int64_t* row_bytes, int32_t* pos_ids_out, void* ws,
+                     size_t ws_bytes, void* stream) {
+  E2S_TRY(check_decide_args(layout, params, q_text, q_row_stride, k, k_row_stride, prior, a_out,
+                            mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
+                            ws, ws_bytes));
+  E2S_TRY(check_compact_args(layout, keep_idx, keep_off, sum_keep, n_tensors, src, dst,
+                             row_bytes));
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (params->flags & E2S_SIMT_SCORE)
-    return from_cuda(launch_score_simt(la, params->score_mode, q_text, q_row_stride, k,
-                                       k_row_stride, a_out, status_word(ws), st));
-  int unsupported = 0;
-  const cudaError_t e = launch_score_tc(la, params->score_mode, q_text, q_row_stride, k,
-                                        k_row_stride, a_out, status_word(ws), st, &unsupported);
-  if (unsupported) return E2S_ERR_UNSUPPORTED;
-  return from_cuda(e);
+  E2S_TRY(run_decide(layout, params, q_text, q_row_stride, k, k_row_stride, cand, prior, a_out,
+                     mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
+                     q_tilde_out, ws, st));
+  if (n_tensors == 0 && !pos_ids_out) return E2S_OK;
+  // the score kernel is an ordinary launch: it starts after all earlier work on
+  // the stream, so the sources are complete before the compaction may start
+  return from_cuda(launch_compact(layout_args(layout), keep_idx, keep_off, sum_keep, n_tensors,
+                                  src, dst, row_bytes, pos_ids_out, status_word(ws), st, 1));
 }
 
 e2s_status e2s_fuse(const e2s_layout* layout, const e2s_params* params, const float* a,
                     const int32_t* cand, const float* prior, float* mass_out, float* fused_out,
                     float* q_out, void* ws, size_t ws_bytes, void* stream) {
-  (void)cand;
   E2S_TRY(check_layout(layout));
   E2S_TRY(check_params(params));
   E2S_TRY(check_ws(layout, ws, ws_bytes));
   if (layout->sum_vis > 0 && (!a || !fused_out || !q_out)) return E2S_ERR_INVALID_ARG;
   if (!aligned16(prior) || !aligned16(mass_out) || !aligned16(fused_out)) return E2S_ERR_ALIGNMENT;
-  return from_cuda(launch_fuse(layout_args(layout), norm_is_softmax(params), params->flags, a,
-                               prior, mass_out, fused_out, q_out, stats_ptr(ws), status_word(ws),
-                               static_cast<cudaStream_t>(stream)));
+  int unsupported = 0;
+  const cudaError_t e = launch_evidence(layout_args(layout), norm_is_softmax(params),
+                                        params->flags, params->lambda, params->G, a, prior, cand,
+                                        mass_out, fused_out, q_out, nullptr, nullptr, nullptr, 0,
+                                        nullptr, 0, status_word(ws),
+                                        static_cast<cudaStream_t>(stream), &unsupported);
+  if (unsupported) return E2S_ERR_UNSUPPORTED;
+  return from_cuda(e);
+}
+
+e2s_status e2s_fuse_select(const e2s_layout* layout, const e2s_params* params, const float* a,
+                           const int32_t* cand, const float* prior, float* mass_out,
+                           float* fused_out, float* q_out, const int32_t* keep_count,
+                           const int32_t* keep_off, int32_t sum_keep, int32_t* keep_idx,
+                           float* q_tilde_out, void* ws, size_t ws_bytes, void* stream) {
+  E2S_TRY(check_layout(layout));
+  E2S_TRY(check_params(params));
+  E2S_TRY(check_ws(layout, ws, ws_bytes));
+  if (layout->sum_vis > 0 && (!a || !fused_out || !q_out)) return E2S_ERR_INVALID_ARG;
+  if (!keep_count || !keep_off || sum_keep < 0) return E2S_ERR_INVALID_ARG;
+  if (sum_keep > 0 && !keep_idx) return E2S_ERR_INVALID_ARG;
+  if (!aligned16(prior) || !aligned16(mass_out) || !aligned16(fused_out)) return E2S_ERR_ALIGNMENT;
+  int unsupported = 0;
+  const cudaError_t e = launch_evidence(layout_args(layout), norm_is_softmax(params),
+                                        params->flags, params->lambda, params->G, a, prior, cand,
+                                        mass_out, fused_out, q_out, q_tilde_out, keep_count,
+                                        keep_off, sum_keep, keep_idx, 1, status_word(ws),
+                                        static_cast<cudaStream_t>(stream), &unsupported);
+  if (unsupported) return E2S_ERR_UNSUPPORTED;
+  return from_cuda(e);
 }
 
 e2s_status e2s_fuse_noalloc(const e2s_layout* layout, const e2s_params* params, const float* a,
@@ -162,19 +297,12 @@ e2s_status e2s_compact(const e2s_layout* layout, const int32_t* keep_idx, const 
                        void* ws, size_t ws_bytes, void* stream) {
   E2S_TRY(check_layout(layout));
   E2S_TRY(check_ws(layout, ws, ws_bytes));
-  if (!keep_off || sum_keep < 0 || sum_keep > layout->sum_vis) return E2S_ERR_SHAPE;
-  if (sum_keep > 0 && !keep_idx) return E2S_ERR_INVALID_ARG;
-  if (n_tensors < 0 || n_tensors > kMaxCompactTensors) return E2S_ERR_INVALID_ARG;
-  if (n_tensors > 0 && (!src || !dst || !row_bytes)) return E2S_ERR_INVALID_ARG;
-  for (int i = 0; i < n_tensors; ++i) {
-    if (!src[i] || !dst[i]) return E2S_ERR_INVALID_ARG;
-    if (row_bytes[i] <= 0) return E2S_ERR_SHAPE;
-    if ((row_bytes[i] & 15) || !aligned16(src[i]) || !aligned16(dst[i])) return E2S_ERR_ALIGNMENT;
-  }
+  E2S_TRY(check_compact_args(layout, keep_idx, keep_off, sum_keep, n_tensors, src, dst,
+                             row_bytes));
   if (n_tensors == 0 && !pos_ids_out) return E2S_OK;
   return from_cuda(launch_compact(layout_args(layout), keep_idx, keep_off, sum_keep, n_tensors,
                                   src, dst, row_bytes, pos_ids_out, status_word(ws),
-                                  static_cast<cudaStream_t>(stream)));
+                                  static_cast<cudaStream_t>(stream), 0));
 }
 
 e2s_status e2s_read_status(const void* ws, void* stream) {

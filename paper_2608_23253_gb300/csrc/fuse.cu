@@ -25,6 +25,8 @@ __global__ void __launch_bounds__(kStatsThreads)
     fuse_stats_kernel(const LayoutArgs la, int softmax, const float* __restrict__ a,
                       float2* __restrict__ stats, uint32_t* status) {
   __shared__ float red[32];
+  pdl_launch_dependents();
+  pdl_wait();
   const int unit = blockIdx.x;
   const int h = unit % la.H;
   const int l = (unit / la.H) % la.L;
@@ -71,6 +73,8 @@ __global__ void __launch_bounds__(kTokenThreads)
                       const float* __restrict__ a, const float2* __restrict__ stats,
                       const float4* __restrict__ prior, float4* __restrict__ mass_out,
                       float4* __restrict__ fused_out, float* __restrict__ q_out) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int gv = blockIdx.x * blockDim.x + threadIdx.x;
   if (gv >= la.sum_vis) return;
   const int b = find_segment(la.vis_off, la.B, gv);
@@ -144,14 +148,14 @@ cudaError_t launch_fuse(const LayoutArgs& la, int norm_softmax, uint32_t flags, 
                         float2* stats, uint32_t* status, cudaStream_t st) {
   if (la.sum_vis == 0) return cudaSuccess;
   const unsigned units = (unsigned)((size_t)la.B * la.L * la.H);
-  fuse_stats_kernel<<<units, kStatsThreads, 0, st>>>(la, norm_softmax, a, stats, status);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_kernel(fuse_stats_kernel, dim3(units), dim3(kStatsThreads), 0, st, 0, true,
+                                la, norm_softmax, a, stats, status);
   if (e != cudaSuccess) return e;
   const unsigned blocks = (unsigned)((la.sum_vis + kTokenThreads - 1) / kTokenThreads);
-  fuse_token_kernel<<<blocks, kTokenThreads, 0, st>>>(
-      la, norm_softmax, flags, a, stats, reinterpret_cast<const float4*>(prior),
-      reinterpret_cast<float4*>(mass_out), reinterpret_cast<float4*>(fused_out), q_out);
-  return cudaGetLastError();
+  return launch_kernel(fuse_token_kernel, dim3(blocks), dim3(kTokenThreads), 0, st, 0, true, la,
+                       norm_softmax, flags, a, static_cast<const float2*>(stats),
+                       reinterpret_cast<const float4*>(prior), reinterpret_cast<float4*>(mass_out),
+                       reinterpret_cast<float4*>(fused_out), q_out);
 }
 
 }  // namespace e2s

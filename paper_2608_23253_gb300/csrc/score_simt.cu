@@ -34,12 +34,17 @@ __device__ __forceinline__ float dot_row(const float* __restrict__ qrow,
 __global__ void __launch_bounds__(kSimtThreads)
     score_simt_kernel(const LayoutArgs la, int mode, const uint16_t* __restrict__ q,
                       int64_t q_stride, const uint16_t* __restrict__ k, int64_t k_stride,
-                      float* __restrict__ a_out, uint32_t* status) {
+                      float* __restrict__ a_out, float4* __restrict__ stats,
+                      uint32_t* counters, uint32_t* status) {
   extern __shared__ float sm[];
   float* Qs = sm;                               // [max_text][128]
   float* lse = Qs + (size_t)la.max_text * 128;  // [max_text]
   float* red = lse + la.max_text;               // [64]
 
+  pdl_launch_dependents();
+  if (counters != nullptr && blockIdx.x == 0)
+    for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
+      counters[i] = 0u;
   const int unit = blockIdx.x;
   const int h = unit % la.H;
   const int l = (unit / la.H) % la.L;
@@ -107,22 +112,34 @@ __global__ void __launch_bounds__(kSimtThreads)
     }
     a_out[((size_t)l * la.H + h) * (size_t)la.sum_vis + v0 + n] = acc * inv_nt;
   }
+  // statistics of this (layer, head)'s visual scores, in a fixed reduction order
+  __syncthreads();
+  const float* arow = a_out + ((size_t)l * la.H + h) * (size_t)la.sum_vis + v0;
+  float ls = 0.f, lm = kNegBig;
+  for (int n = threadIdx.x; n < NV; n += blockDim.x) {
+    ls += arow[n];
+    lm = fmaxf(lm, arow[n] * 1.4426950408889634f);
+  }
+  const float S_ = block_reduce(ls, [](float x, float y) { return x + y; }, red);
+  const float M_ = block_reduce(lm, [](float x, float y) { return fmaxf(x, y); }, red);
+  float le = 0.f;
+  for (int n = threadIdx.x; n < NV; n += blockDim.x)
+    le += fast_ex2(fmaf(arow[n], 1.4426950408889634f, -M_));
+  const float E_ = block_reduce(le, [](float x, float y) { return x + y; }, red);
+  if (threadIdx.x == 0) stats[((size_t)b * la.L + l) * la.H + h] = stats_entry(S_, M_, E_);
 }
 
 }  // namespace
 
 cudaError_t launch_score_simt(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
-                              const void* k, int64_t k_stride, float* a_out, uint32_t* status,
-                              cudaStream_t st) {
+                              const void* k, int64_t k_stride, float* a_out, float4* stats,
+                              uint32_t* counters, uint32_t* status, cudaStream_t st) {
   const size_t smem = ((size_t)la.max_text * 129 + 64) * sizeof(float);
-  cudaError_t e = cudaFuncSetAttribute(score_simt_kernel,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
   const unsigned grid = (unsigned)((size_t)la.B * la.L * la.H);
-  score_simt_kernel<<<grid, kSimtThreads, smem, st>>>(la, mode, static_cast<const uint16_t*>(q),
-                                                      q_stride, static_cast<const uint16_t*>(k),
-                                                      k_stride, a_out, status);
-  return cudaGetLastError();
+  return launch_kernel(score_simt_kernel, dim3(grid), dim3(kSimtThreads), smem, st, 0, false, la,
+                       mode, static_cast<const uint16_t*>(q), q_stride,
+                       static_cast<const uint16_t*>(k), k_stride, a_out, stats, counters,
+                       status);
 }
 
 }  // namespace e2s

@@ -2,26 +2,30 @@
 // with TMA-staged bf16 K tiles (Sec. 3.1 Eq. 1 and its causal-prefix
 // probability reading).
 //
-// Work unit: (image b, layer l, kv head g, group of query heads).  A unit's
-// keys are cut into 128-key tiles; a cluster of `cluster` CTAs splits the
-// tiles, each CTA keeping its tiles resident in shared memory.
+// Work unit: (image b, layer l, kv head g, group of query heads).  The unit's
+// keys are cut into 128-key tiles and split over a thread-block cluster; each
+// CTA multiplies its tiles once and keeps every logit in TMEM:
 //
-//   MMA  D[key][col] = K_tile[key][:] . Q[col][:]       (M = 128 keys,
-//        N = padded text rows of one query head, K = d = 128 in 8 steps)
-//        A = K tile, B = text queries, both K-major with the 128-byte swizzle,
-//        fp32 accumulator in TMEM (two buffers).
-//   CAUSAL_PROB phase 1: every epilogue thread owns one key (TMEM lane); per
-//        16-column chunk a butterfly reduce-scatter over the warp's 32 lanes
-//        turns 32 keys x 16 text rows into per-row online-softmax partials
-//        (max, sum) in the log2 domain; partials are merged per warp, per CTA,
-//        and then across the cluster through distributed shared memory,
-//        giving each text row's log-sum-exp over its whole causal prefix.
-//   phase 2: the visual tiles are multiplied again from the resident shared
-//        memory copy; each thread sums exp2(s - lse) over the text rows of
-//        its key and writes a = sum / N_T (EQ1 mode: the mean logit).
+//   MMA   D[key][col] = K_tile[key][:] . Q[col][:]   (M = 128 keys, N = padded
+//         text rows of one query head, K = d = 128 in 8 steps), A = K tile and
+//         B = text queries, both K-major with the 128-byte swizzle; tile i of
+//         the CTA accumulates into TMEM columns [i*ncs, (i+1)*ncs).
+//   pass A (CAUSAL_PROB)  per-text-row maximum over this CTA's visible keys:
+//         a butterfly reduce-scatter over the warp's 32 lanes per 16-column
+//         chunk, then over the four TMEM lane quarters in shared memory.
+//   pass B  e = exp2(s - M) for every visible logit (one exp2 per logit),
+//         written back into TMEM for the visual tiles, and the per-row sum L.
+//   cluster exchange of (M, L) through distributed shared memory; every CTA
+//         forms the row's log-sum-exp and a per-row weight
+//         w = exp2(M_cta - lse) / N_T.
+//   pass C  a[key] = sum_t e[key][t] * w[t] over the text rows (FMA only);
+//         EQ1 mode: a = sum_t s[key][t] / (sqrt(d) N_T) straight from TMEM.
 //
-// Warp roles (192 threads): warp 0 TMA producer, warp 1 TMEM allocator and
-// MMA issuer, warps 2-5 epilogue (TMEM lane quarter = warp % 4).
+// Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator and
+// MMA issuer, warps 2-9 epilogue.  Epilogue warp w reads TMEM lane quarter
+// w % 4; in passes A and B it owns the 16-column chunks of parity (w - 2) / 4
+// across all of the CTA's tiles (running max / sum per lane, one butterfly per
+// chunk), in pass C the tiles of that parity.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -36,9 +40,11 @@ namespace {
 constexpr int kTileKeys = 128;
 constexpr int kHalfBytes = kTileKeys * 128;   // 128 rows x 64 bf16 (one swizzle span)
 constexpr int kTileBytes = 2 * kHalfBytes;    // 128 keys x 128 dims
-constexpr int kEpiWarps = 4;
-constexpr int kThreads = 64 + 32 * kEpiWarps;
+constexpr int kEpiWarps = 8;
+constexpr int kEpiThreads = 32 * kEpiWarps;
+constexpr int kThreads = 64 + kEpiThreads;
 constexpr int kQBoxRows = 16;
+constexpr int kMaxCluster = 16;
 constexpr uint64_t kWaitNs = 1000000000ull;        // first bounded wait: 1 s
 constexpr uint64_t kWaitNsAfterFault = 1000000ull; // later waits after a timeout: 1 ms
 
@@ -55,11 +61,13 @@ struct TcArgs {
   float scale;         // 1 / sqrt(d)
   uint32_t tmem_cols;
   float* a_out;
+  float4* stats;        // per (image, layer, head) statistics of the visual scores
+  uint32_t* counters;   // nullable: decision scratch to zero
   uint32_t* status;
 };
 
 struct SmemPlan {
-  uint32_t q, k, bars, slot, wstats, part, colv, total;
+  uint32_t q, k, bars, slot, pmax, psum, cm, part, colw, asm_, sred, spart, total;
 };
 
 __host__ __device__ inline SmemPlan smem_plan(int hpc, int ntp_max, int tpc) {
@@ -68,44 +76,45 @@ __host__ __device__ inline SmemPlan smem_plan(int hpc, int ntp_max, int tpc) {
   s.q = 0;
   s.k = 2u * ncs * 128u;
   s.bars = s.k + (uint32_t)tpc * kTileBytes;
-  s.slot = s.bars + 8u * (uint32_t)(5 + tpc);
-  s.wstats = (s.slot + 16u + 15u) & ~15u;
-  s.part = s.wstats + (uint32_t)kEpiWarps * ncs * 8u;
-  s.colv = s.part + ncs * 8u;
-  s.total = s.colv + ncs * 4u;
+  s.slot = s.bars + 8u * (uint32_t)(1 + 2 * tpc);
+  s.pmax = (s.slot + 16u + 15u) & ~15u;       // [4 lane quarters][ncs] float
+  s.psum = s.pmax + 4u * ncs * 4u;            // [4 lane quarters][ncs] float
+  s.cm = s.psum + 4u * ncs * 4u;              // [ncs] float: CTA max (log2 units)
+  s.part = s.cm + ncs * 4u;                   // [ncs] float2: (M, L) for the cluster
+  s.colw = s.part + ncs * 8u;                 // [ncs] float: pass-C weights
+  s.asm_ = s.colw + ncs * 4u;                 // [hpc][tpc*128] float: this CTA's scores
+  s.sred = s.asm_ + (uint32_t)hpc * (uint32_t)tpc * 128u * 4u;  // [8 warps] float2
+  s.spart = s.sred + 8u * 8u;                 // [hpc] float4: CTA statistics
+  s.total = s.spart + (uint32_t)hpc * 16u;
   return s;
 }
 
-// One butterfly step of the reduce-scatter: keep W of the 2W live entries
-// (upper half if `hi`), send the other W to the partner lane (xor MASK) and
-// merge what comes back.
-template <int W, int MASK>
-__device__ __forceinline__ void rs_step(float (&m)[16], float (&s)[16], bool hi) {
+// Butterfly reduce-scatter of 16 values over the 32 lanes of a warp: on
+// return lane L holds, in x[0], column L >> 1 reduced over all 32 lanes.
+template <int W, int MASK, class Op>
+__device__ __forceinline__ void rs_step(float (&x)[16], bool hi, Op op) {
 #pragma unroll
   for (int i = 0; i < W; ++i) {
-    const float send_m = hi ? m[i] : m[i + W];
-    const float send_s = hi ? s[i] : s[i + W];
-    float keep_m = hi ? m[i + W] : m[i];
-    float keep_s = hi ? s[i + W] : s[i];
-    const float rm = __shfl_xor_sync(0xffffffffu, send_m, MASK);
-    const float rs = __shfl_xor_sync(0xffffffffu, send_s, MASK);
-    lse_merge(keep_m, keep_s, rm, rs);
-    m[i] = keep_m;
-    s[i] = keep_s;
+    const float send = hi ? x[i] : x[i + W];
+    const float keep = hi ? x[i + W] : x[i];
+    x[i] = op(keep, __shfl_xor_sync(0xffffffffu, send, MASK));
   }
 }
-
-// 32 lanes x 16 columns of (max, sum) partials -> lane L holds column L >> 1
-// reduced over all 32 lanes (lanes L and L ^ 1 hold the same result).
-__device__ __forceinline__ void reduce_scatter16(float (&m)[16], float (&s)[16], int lane) {
-  rs_step<8, 16>(m, s, lane & 16);
-  rs_step<4, 8>(m, s, lane & 8);
-  rs_step<2, 4>(m, s, lane & 4);
-  rs_step<1, 2>(m, s, lane & 2);
-  const float rm = __shfl_xor_sync(0xffffffffu, m[0], 1);
-  const float rs = __shfl_xor_sync(0xffffffffu, s[0], 1);
-  lse_merge(m[0], s[0], rm, rs);
+template <class Op>
+__device__ __forceinline__ float reduce_scatter16(float (&x)[16], int lane, Op op) {
+  rs_step<8, 16>(x, lane & 16, op);
+  rs_step<4, 8>(x, lane & 8, op);
+  rs_step<2, 4>(x, lane & 4, op);
+  rs_step<1, 2>(x, lane & 2, op);
+  return op(x[0], __shfl_xor_sync(0xffffffffu, x[0], 1));
 }
+
+struct MaxOp {
+  __device__ __forceinline__ float operator()(float a, float b) const { return fmaxf(a, b); }
+};
+struct AddOp {
+  __device__ __forceinline__ float operator()(float a, float b) const { return a + b; }
+};
 
 __global__ void __launch_bounds__(kThreads, 2)
     score_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
@@ -119,17 +128,25 @@ __global__ void __launch_bounds__(kThreads, 2)
   uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + plan.bars);
   uint64_t* k_full = q_full + 1;
   uint64_t* mma_done = k_full + p.tpc;
-  uint64_t* tmem_empty = mma_done + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + plan.slot);
-  float2* warp_stats = reinterpret_cast<float2*>(smem + plan.wstats);
-  float2* cta_part = reinterpret_cast<float2*>(smem + plan.part);
-  float* colv = reinterpret_cast<float*>(smem + plan.colv);
+  float* pmax = reinterpret_cast<float*>(smem + plan.pmax);
+  float* psum = reinterpret_cast<float*>(smem + plan.psum);
+  float* cm = reinterpret_cast<float*>(smem + plan.cm);
+  float2* part = reinterpret_cast<float2*>(smem + plan.part);
+  float* colw = reinterpret_cast<float*>(smem + plan.colw);
+  float* a_sm = reinterpret_cast<float*>(smem + plan.asm_);
+  float2* sred = reinterpret_cast<float2*>(smem + plan.sred);
+  float4* spart = reinterpret_cast<float4*>(smem + plan.spart);
 
   const LayoutArgs& la = p.la;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = ptx::cluster_ctarank();
   const int ncs = p.hpc * p.ntp_max;
   const uint32_t q_half = (uint32_t)ncs * 128u;
+  pdl_launch_dependents();
+  if (p.counters != nullptr && blockIdx.x == 0)
+    for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
+      p.counters[i] = 0u;
 
   // ---- unit decomposition: (b, l, kv head, head group)
   const int unit = blockIdx.x / p.cluster;
@@ -175,16 +192,13 @@ __global__ void __launch_bounds__(kThreads, 2)
       vl = i + 1;
     }
   }
-  const int n1 = causal ? nt : 0;
-  const int njobs = n1 + (vl - vf);
 
   // ---- setup: barriers, TMEM
   if (warp == 0 && lane == 0) {
     ptx::mbar_init(q_full, 1);
-    for (int i = 0; i < p.tpc; ++i) ptx::mbar_init(k_full + i, 1);
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < p.tpc; ++i) {
+      ptx::mbar_init(k_full + i, 1);
       ptx::mbar_init(mma_done + i, 1);
-      ptx::mbar_init(tmem_empty + i, kEpiWarps);
     }
     ptx::fence_barrier_init();
     ptx::fence_proxy_async_smem();
@@ -200,7 +214,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 
   if (warp == 0) {
     // ================= TMA producer
-    if (lane == 0 && njobs > 0) {
+    if (lane == 0 && nt > 0) {
       ptx::mbar_arrive_expect_tx(q_full, 2u * (uint32_t)(nh * ntp) * 128u);
       for (int hh = 0; hh < nh; ++hh)
         for (int half = 0; half < 2; ++half)
@@ -222,142 +236,222 @@ __global__ void __launch_bounds__(kThreads, 2)
     ptx::cluster_arrive();
     ptx::cluster_wait();
   } else if (warp == 1) {
-    // ================= MMA issuer (one thread)
-    const uint32_t idesc = ptx::idesc_bf16_f32(128, ntp);
-    auto issue = [&](int j, int tile) {
-      const int buf = j & 1, use = j >> 1;
-      if (!ptx::mbar_wait(k_full + tile, 0, limit, p.status)) limit = kWaitNsAfterFault;
-      if (use > 0 && !ptx::mbar_wait(tmem_empty + buf, (use - 1) & 1, limit, p.status))
-        limit = kWaitNsAfterFault;
-      ptx::tc_fence_after();
-      const uint32_t a_base = ptx::smem_addr(k_sm + tile * kTileBytes);
-      const uint32_t b_base = ptx::smem_addr(q_sm);
-      for (int hh = 0; hh < nh; ++hh) {
-        const uint32_t d = tmem + (uint32_t)(buf * ncs + hh * p.ntp_max);
-#pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-          const uint32_t half = ks >> 2, kk = ks & 3;
-          const uint64_t ad = ptx::sdesc_sw128(a_base + half * kHalfBytes + kk * 32u);
-          const uint64_t bd = ptx::sdesc_sw128(b_base + half * q_half +
-                                               (uint32_t)(hh * p.ntp_max) * 128u + kk * 32u);
-          ptx::mma_bf16(d, ad, bd, idesc, ks > 0 ? 1u : 0u);
-        }
-      }
-      ptx::mma_commit(mma_done + buf);
-    };
-    if (lane == 0 && njobs > 0) {
+    // ================= MMA issuer (one thread): every tile once, own TMEM columns
+    if (lane == 0 && nt > 0) {
+      const uint32_t idesc = ptx::idesc_bf16_f32(128, ntp);
       if (!ptx::mbar_wait(q_full, 0, limit, p.status)) limit = kWaitNsAfterFault;
-      for (int j = 0; j < n1; ++j) issue(j, j);
+      const uint32_t b_base = ptx::smem_addr(q_sm);
+      for (int i = 0; i < nt; ++i) {
+        if (!ptx::mbar_wait(k_full + i, 0, limit, p.status)) limit = kWaitNsAfterFault;
+        ptx::tc_fence_after();
+        const uint32_t a_base = ptx::smem_addr(k_sm + i * kTileBytes);
+        for (int hh = 0; hh < nh; ++hh) {
+          const uint32_t d = tmem + (uint32_t)(i * ncs + hh * p.ntp_max);
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks) {
+            const uint32_t half = ks >> 2, kk = ks & 3;
+            const uint64_t ad = ptx::sdesc_sw128(a_base + half * kHalfBytes + kk * 32u);
+            const uint64_t bd = ptx::sdesc_sw128(b_base + half * q_half +
+                                                 (uint32_t)(hh * p.ntp_max) * 128u + kk * 32u);
+            ptx::mma_bf16(d, ad, bd, idesc, ks > 0 ? 1u : 0u);
+          }
+        }
+        ptx::mma_commit(mma_done + i);
+      }
     }
     __syncwarp();
     ptx::cluster_arrive();
-    if (lane == 0)
-      for (int j = n1; j < njobs; ++j) issue(j, vf + (j - n1));
-    __syncwarp();
     ptx::cluster_wait();
   } else {
-    // ================= epilogue (4 warps, one TMEM lane quarter each)
+    // ================= epilogue (8 warps)
     const int ew = warp - 2;
-    const int q4 = warp & 3;
+    const int q4 = warp & 3;       // TMEM lane quarter
+    const int par = ew >> 2;       // chunk parity (passes A, B) / tile parity (pass C)
     const int row = q4 * 32 + lane;
     const uint32_t lane_base = (uint32_t)(q4 * 32) << 16;
     const int et = threadIdx.x - 64;
-    float2* my_stats = warp_stats + ew * ncs;
+    const int lim = S + NV;        // text row t sees key k iff k <= lim + t
+    const int cpb = ntp >> 4;      // chunks per head
 
     if (causal) {
-      for (int c = lane; c < ncs; c += 32) my_stats[c] = make_float2(kNegBig, 0.f);
-      __syncwarp();
-      for (int j = 0; j < n1; ++j) {
-        const int buf = j & 1;
-        if (!ptx::mbar_wait(mma_done + buf, (j >> 1) & 1, limit, p.status))
-          limit = kWaitNsAfterFault;
-        ptx::tc_fence_after();
-        const int key = key_base + kTileKeys * (ft + j) + row;
-        const int last_text = key - (S + NV);  // row t sees this key iff t >= last_text
-        for (int hh = 0; hh < nh; ++hh) {
-          for (int c16 = 0; c16 < ntp; c16 += 16) {
-            float v[16], m[16], s[16];
-            ptx::tmem_ld16(tmem + lane_base + (uint32_t)(buf * ncs + hh * p.ntp_max + c16), v);
+      // ---- pass A: per-column maximum of the visible raw logits
+      for (int i = 0; i < nt; ++i)
+        if (!ptx::mbar_wait(mma_done + i, 0, limit, p.status)) limit = kWaitNsAfterFault;
+      ptx::tc_fence_after();
+      for (int hh = 0; hh < nh; ++hh) {
+        for (int c = par; c < cpb; c += 2) {
+          const int c16 = c * 16;
+          const int col = hh * p.ntp_max + c16;
+          float mx[16];
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const int t = c16 + i;
-              const bool valid = t < NT && t >= last_text;
-              m[i] = valid ? v[i] * p.scale_log2 : kNegBig;
-              s[i] = valid ? 1.f : 0.f;
-            }
-            reduce_scatter16(m, s, lane);
-            if ((lane & 1) == 0) {
-              float2 st = my_stats[hh * p.ntp_max + c16 + (lane >> 1)];
-              lse_merge(st.x, st.y, m[0], s[0]);
-              my_stats[hh * p.ntp_max + c16 + (lane >> 1)] = st;
+          for (int j = 0; j < 16; ++j) mx[j] = kNegBig;
+          for (int i = 0; i < nt; ++i) {
+            const int lo = max(key_base + kTileKeys * (ft + i) + row - lim, 0);
+            float x[16];
+            ptx::tmem_ld16(tmem + lane_base + (uint32_t)(i * ncs + col), x);
+            if (lo <= c16 && c16 + 16 <= NT) {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) mx[j] = fmaxf(mx[j], x[j]);
+            } else {
+#pragma unroll
+              for (int j = 0; j < 16; ++j)
+                if (c16 + j >= lo && c16 + j < NT) mx[j] = fmaxf(mx[j], x[j]);
             }
           }
+          const float m = reduce_scatter16(mx, lane, MaxOp());
+          if ((lane & 1) == 0) pmax[q4 * ncs + col + (lane >> 1)] = m;
         }
-        ptx::tc_fence_before();
-        __syncwarp();
-        if (lane == 0) ptx::mbar_arrive(tmem_empty + buf);
       }
-      ptx::named_bar(1, 32 * kEpiWarps);
-      for (int c = et; c < ncs; c += 32 * kEpiWarps) {
-        float2 acc = warp_stats[c];
-        for (int w = 1; w < kEpiWarps; ++w) {
-          const float2 o = warp_stats[w * ncs + c];
-          lse_merge(acc.x, acc.y, o.x, o.y);
+      ptx::named_bar(1, kEpiThreads);
+      for (int c = et; c < ncs; c += kEpiThreads) {
+        const float m = fmaxf(fmaxf(pmax[c], pmax[ncs + c]), fmaxf(pmax[2 * ncs + c], pmax[3 * ncs + c]));
+        cm[c] = m > 0.5f * kNegBig ? m * p.scale_log2 : kNegBig;
+      }
+      ptx::named_bar(1, kEpiThreads);
+      // ---- pass B: e = exp2(s - M), stored back for visual tiles; row sums
+      for (int hh = 0; hh < nh; ++hh) {
+        for (int c = par; c < cpb; c += 2) {
+          const int c16 = c * 16;
+          const int col = hh * p.ntp_max + c16;
+          float mv[16], sm[16];
+          const float4* cm4 = reinterpret_cast<const float4*>(cm + col);
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            const float4 c4 = cm4[v];
+            mv[4 * v] = c4.x; mv[4 * v + 1] = c4.y; mv[4 * v + 2] = c4.z; mv[4 * v + 3] = c4.w;
+          }
+#pragma unroll
+          for (int j = 0; j < 16; ++j) sm[j] = 0.f;
+          for (int i = 0; i < nt; ++i) {
+            const int lo = max(key_base + kTileKeys * (ft + i) + row - lim, 0);
+            const uint32_t ta = tmem + lane_base + (uint32_t)(i * ncs + col);
+            float x[16];
+            ptx::tmem_ld16(ta, x);
+            if (lo <= c16 && c16 + 16 <= NT) {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) x[j] = fast_ex2(fmaf(x[j], p.scale_log2, -mv[j]));
+            } else {
+#pragma unroll
+              for (int j = 0; j < 16; ++j)
+                x[j] = (c16 + j >= lo && c16 + j < NT) ? fast_ex2(fmaf(x[j], p.scale_log2, -mv[j]))
+                                                       : 0.f;
+            }
+            if (i >= vf && i < vl) ptx::tmem_st16(ta, x);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) sm[j] += x[j];
+          }
+          const float sum = reduce_scatter16(sm, lane, AddOp());
+          if ((lane & 1) == 0) psum[q4 * ncs + col + (lane >> 1)] = sum;
         }
-        cta_part[c] = acc;
       }
+      ptx::tmem_wait_st();
+      ptx::tc_fence_before();
+      ptx::named_bar(1, kEpiThreads);
+      ptx::tc_fence_after();
+      for (int c = et; c < ncs; c += kEpiThreads)
+        part[c] = make_float2(cm[c], ((psum[c] + psum[ncs + c]) + psum[2 * ncs + c]) + psum[3 * ncs + c]);
     }
     ptx::cluster_arrive();
     ptx::cluster_wait();
-    // per-column constants of phase 2
-    for (int c = et; c < ncs; c += 32 * kEpiWarps) {
+    // ---- per-column weights of pass C
+    for (int c = et; c < ncs; c += kEpiThreads) {
       const int t = c % p.ntp_max;
       if (causal) {
+        float2 o[kMaxCluster];
+#pragma unroll
+        for (int r = 0; r < kMaxCluster; ++r)
+          if (r < p.cluster) o[r] = ptx::ld_dsmem_f2(part + c, (uint32_t)r);
         float M = kNegBig, Ls = 0.f;
-        for (int r = 0; r < p.cluster; ++r) {
-          const float2 o = ptx::ld_dsmem_f2(cta_part + c, (uint32_t)r);
-          lse_merge(M, Ls, o.x, o.y);
-        }
-        colv[c] = (t < NT && Ls > 0.f) ? M + log2f(Ls) : __int_as_float(0x7f800000);
+#pragma unroll
+        for (int r = 0; r < kMaxCluster; ++r)
+          if (r < p.cluster) lse_merge(M, Ls, o[r].x, o[r].y);
+        const float lse = M + log2f(Ls);
+        colw[c] = (t < NT && Ls > 0.f) ? fast_ex2(part[c].x - lse) / (float)NT : 0.f;
       } else {
-        colv[c] = (t < NT) ? 1.f : 0.f;
+        colw[c] = (t < NT) ? p.scale / (float)NT : 0.f;
       }
     }
-    ptx::named_bar(1, 32 * kEpiWarps);
-    const float out_scale = causal ? 1.f / (float)NT : p.scale / (float)NT;
-    for (int j = n1; j < njobs; ++j) {
-      const int buf = j & 1;
-      if (!ptx::mbar_wait(mma_done + buf, (j >> 1) & 1, limit, p.status))
-        limit = kWaitNsAfterFault;
-      ptx::tc_fence_after();
-      const int tile = vf + (j - n1);
-      const int key = key_base + kTileKeys * (ft + tile) + row;
+    ptx::named_bar(1, kEpiThreads);
+    // ---- pass C: a[key] = sum_t e[key][t] w[t] for the visual tiles
+    for (int i = vf + ((vf & 1) != par ? 1 : 0); i < vl; i += 2) {
+      if (!causal) {
+        if (!ptx::mbar_wait(mma_done + i, 0, limit, p.status)) limit = kWaitNsAfterFault;
+        ptx::tc_fence_after();
+      }
+      const int key = key_base + kTileKeys * (ft + i) + row;
       const bool vis = key >= S && key < S + NV;
       for (int hh = 0; hh < nh; ++hh) {
-        float acc = 0.f;
+        float acc0 = 0.f, acc1 = 0.f;
         for (int c16 = 0; c16 < ntp; c16 += 16) {
-          float v[16];
-          ptx::tmem_ld16(tmem + lane_base + (uint32_t)(buf * ncs + hh * p.ntp_max + c16), v);
-          const float* cv = colv + hh * p.ntp_max + c16;
-          if (causal) {
+          const int col = hh * p.ntp_max + c16;
+          float x[16];
+          ptx::tmem_ld16(tmem + lane_base + (uint32_t)(i * ncs + col), x);
+          const float4* w4 = reinterpret_cast<const float4*>(colw + col);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) acc += exp2f(fmaf(v[i], p.scale_log2, -cv[i]));
-          } else {
-#pragma unroll
-            for (int i = 0; i < 16; ++i) acc = fmaf(v[i], cv[i], acc);
+          for (int v = 0; v < 4; ++v) {
+            const float4 w = w4[v];
+            acc0 = fmaf(x[4 * v], w.x, acc0);
+            acc1 = fmaf(x[4 * v + 1], w.y, acc1);
+            acc0 = fmaf(x[4 * v + 2], w.z, acc0);
+            acc1 = fmaf(x[4 * v + 3], w.w, acc1);
           }
         }
+        a_sm[hh * p.tpc * kTileKeys + i * kTileKeys + row] = acc0 + acc1;
         if (vis)
           p.a_out[((size_t)l * la.H + h0 + hh) * (size_t)la.sum_vis + v0 + (key - S)] =
-              acc * out_scale;
+              acc0 + acc1;
       }
-      ptx::tc_fence_before();
-      __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(tmem_empty + buf);
+    }
+    // ---- this CTA's share of the (layer, head) statistics of the visual scores
+    ptx::named_bar(1, kEpiThreads);
+    const int kb0 = key_base + kTileKeys * ft;
+    const int i_lo = max(S, kb0) - kb0;
+    const int i_hi = max(min(S + NV, kb0 + kTileKeys * nt) - kb0, i_lo);
+    for (int hh = 0; hh < nh; ++hh) {
+      const float* ah = a_sm + hh * p.tpc * kTileKeys;
+      float ls = 0.f, lm = kNegBig;
+      for (int x = i_lo + et; x < i_hi; x += kEpiThreads) {
+        ls += ah[x];
+        lm = fmaxf(lm, ah[x] * 1.4426950408889634f);
+      }
+      ls = warp_reduce(ls, [](float u, float v) { return u + v; });
+      lm = warp_reduce(lm, [](float u, float v) { return fmaxf(u, v); });
+      if (lane == 0) sred[ew] = make_float2(ls, lm);
+      ptx::named_bar(1, kEpiThreads);
+      float Sa = 0.f, Ma = kNegBig;
+      for (int w = 0; w < kEpiWarps; ++w) {
+        Sa += sred[w].x;
+        Ma = fmaxf(Ma, sred[w].y);
+      }
+      ptx::named_bar(1, kEpiThreads);
+      float le = 0.f;
+      for (int x = i_lo + et; x < i_hi; x += kEpiThreads)
+        le += fast_ex2(fmaf(ah[x], 1.4426950408889634f, -Ma));
+      le = warp_reduce(le, [](float u, float v) { return u + v; });
+      if (lane == 0) sred[ew] = make_float2(le, 0.f);
+      ptx::named_bar(1, kEpiThreads);
+      if (et == 0) {
+        float Ea = 0.f;
+        for (int w = 0; w < kEpiWarps; ++w) Ea += sred[w].x;
+        spart[hh] = make_float4(Sa, Ma, Ea, 0.f);
+      }
+      ptx::named_bar(1, kEpiThreads);
     }
   }
 
-  // ---- teardown: peers may still read cta_part until everyone is here
+  // ---- teardown: peers may still read `part`; rank 0 merges the statistics
+  ptx::cluster_arrive();
+  ptx::cluster_wait();
+  if (rank == 0 && ok && threadIdx.x >= 64 && threadIdx.x - 64 < nh) {
+    const int hh = threadIdx.x - 64;
+    float Sa = 0.f, Ma = kNegBig, Ea = 0.f;
+    for (int r = 0; r < p.cluster; ++r) {
+      const float4 o = ptx::ld_dsmem_f4(spart + hh, (uint32_t)r);
+      Sa += o.x;
+      lse_merge(Ma, Ea, o.y, o.z);
+    }
+    p.stats[((size_t)b * la.L + l) * la.H + h0 + hh] = stats_entry(Sa, Ma, Ea);
+  }
   ptx::cluster_arrive();
   ptx::cluster_wait();
   ptx::tc_fence_before();
@@ -388,8 +482,10 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
+}  // namespace
+
 // 3-D map over rows of (heads x 128) bf16: dims (128, heads, rows), box (64, 1, box_rows).
-bool make_map(CUtensorMap* map, const void* base, int heads, int64_t rows, int64_t row_stride_el,
+bool make_score_map(CUtensorMap* map, const void* base, int heads, int64_t rows, int64_t row_stride_el,
               int box_rows) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
@@ -402,12 +498,15 @@ bool make_map(CUtensorMap* map, const void* base, int heads, int64_t rows, int64
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-}  // namespace
 
 cudaError_t launch_score_tc(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
-                            const void* k, int64_t k_stride, float* a_out, uint32_t* status,
-                            cudaStream_t st, int* unsupported) {
+                            const void* k, int64_t k_stride, float* a_out, float4* stats,
+                            uint32_t* counters, uint32_t* status, cudaStream_t st,
+                            int* unsupported) {
   *unsupported = 0;
+  if (score_unit_fits(la, mode))
+    return launch_score_unit(la, mode, q, q_stride, k, k_stride, a_out, stats, counters, status,
+                             st);
   TcArgs p;
   p.la = la;
   p.group = la.H / la.H_kv;
@@ -420,21 +519,28 @@ cudaError_t launch_score_tc(const LayoutArgs& la, int mode, const void* q, int64
   p.hpc = std::max(1, std::min(p.group, 256 / p.ntp_max));
   p.groups_per_kv = (p.group + p.hpc - 1) / p.hpc;
   const int ncs = p.hpc * p.ntp_max;
-  uint32_t cols = 32;
-  while ((int)cols < 2 * ncs) cols <<= 1;
-  p.tmem_cols = cols;
   const int span = (mode == E2S_SCORE_CAUSAL_PROB) ? la.max_T : la.max_vis;
   const int max_tiles = (span + kTileKeys - 1) / kTileKeys;
   if (max_tiles == 0 || la.sum_vis == 0) return cudaSuccess;
-  p.tpc = std::min(2, max_tiles);
+  const int tpc_tmem = std::max(1, 512 / ncs);  // every tile's logits stay in TMEM
+  p.tpc = std::min({2, max_tiles, tpc_tmem});
   p.cluster = (max_tiles + p.tpc - 1) / p.tpc;
-  while (p.cluster > 8) {
+  while (p.cluster > kMaxCluster && p.tpc < tpc_tmem) {
     ++p.tpc;
     p.cluster = (max_tiles + p.tpc - 1) / p.tpc;
   }
+  if (p.cluster > kMaxCluster) {
+    *unsupported = 1;
+    return cudaSuccess;
+  }
+  uint32_t cols = 32;
+  while ((int)cols < p.tpc * ncs) cols <<= 1;
+  p.tmem_cols = cols;
   p.scale = 1.0f / sqrtf(128.0f);
   p.scale_log2 = 1.4426950408889634f / sqrtf(128.0f);
   p.a_out = a_out;
+  p.stats = stats;
+  p.counters = counters;
   p.status = status;
 
   int dev = 0, smem_sm = 0, smem_optin = 0, reserved = 0;
@@ -455,25 +561,12 @@ cudaError_t launch_score_tc(const LayoutArgs& la, int mode, const void* q, int64
     return cudaSuccess;
   }
   CUtensorMap tmQ, tmK;
-  if (!make_map(&tmQ, q, la.H, (int64_t)la.L * la.sum_text, q_stride, kQBoxRows) ||
-      !make_map(&tmK, k, la.H_kv, (int64_t)la.L * la.sum_T, k_stride, kTileKeys))
+  if (!make_score_map(&tmQ, q, la.H, (int64_t)la.L * la.sum_text, q_stride, kQBoxRows) ||
+      !make_score_map(&tmK, k, la.H_kv, (int64_t)la.L * la.sum_T, k_stride, kTileKeys))
     return cudaErrorInvalidValue;
-  e = cudaFuncSetAttribute(score_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
   const long long units = (long long)la.B * la.L * la.H_kv * p.groups_per_kv;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)(units * p.cluster));
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = p.cluster;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, score_tc_kernel, tmQ, tmK, p);
+  return launch_kernel(score_tc_kernel, dim3((unsigned)(units * p.cluster)), dim3(kThreads), smem,
+                       st, p.cluster, false, tmQ, tmK, p);
 }
 
 }  // namespace e2s

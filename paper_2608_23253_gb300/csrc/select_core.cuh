@@ -1,0 +1,245 @@
+// Spatial novelty and global Top-K of one image, run by a whole CTA
+// (Sec. 4.3, Eqs. 20-23):
+//   1. cell representative: per occupied G x G cell, arg-max of q with ties
+//      to the lower index, as a 64-bit atomicMax of (ordered q bits, ~n);
+//   2. q~ = (1 - lambda) q + lambda b;
+//   3. exact K-th largest q~ by a 4-pass 8-bit radix select over the ordered
+//      bit patterns (histogram in shared memory, digit found by a warp scan);
+//   4. emission in ascending index order with block-wide prefix counts; among
+//      tokens equal to the threshold the lowest indices are kept.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "device_common.cuh"
+
+namespace e2s {
+
+constexpr int kMaxCells = 64;
+
+struct SelectSmem {
+  unsigned long long cell_best[kMaxCells];
+  uint32_t hist[3][256];   // one per radix pass, rotating (zeroed two passes ahead)
+  uint32_t warp_tot[32];
+};
+
+// Exclusive prefix count of `flag` over the block (in thread order) and the
+// block total.  Every thread of the block must call it.
+__device__ __forceinline__ uint32_t block_excl_count(bool flag, uint32_t* warp_tot,
+                                                     uint32_t& total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const uint32_t bal = __ballot_sync(0xffffffffu, flag);
+  const uint32_t in_warp = __popc(bal & ((1u << lane) - 1u));
+  __syncthreads();
+  if (lane == 0) warp_tot[warp] = __popc(bal);
+  __syncthreads();
+  uint32_t before = 0, all = 0;
+  for (int w = 0; w < nw; ++w) {
+    const uint32_t c = warp_tot[w];
+    before += (w < warp) ? c : 0u;
+    all += c;
+  }
+  total = all;
+  return before + in_warp;
+}
+
+__device__ __forceinline__ int cell_id(int r, int gh, int gw, int G) {
+  const int i = r / gw, j = r - (r / gw) * gw;
+  return (i * G / gh) * G + (j * G / gw);
+}
+
+// Cell of image-local slot n: its original raster index (cand, when given)
+// mapped to the G x G grid of cells.  An out-of-range candidate raises
+// E2S_ERR_SHAPE and is clamped.
+__device__ __forceinline__ int token_cell(const int32_t* cand, int n, int gh, int gw, int G,
+                                          uint32_t* status) {
+  int r = cand ? __ldg(cand + n) : n;
+  if (r < 0 || r >= gh * gw) {
+    E2S_DEV_FLAG(status, E2S_ERR_SHAPE);
+    r = min(max(r, 0), gh * gw - 1);
+  }
+  return cell_id(r, gh, gw, G);
+}
+
+// Arg-max key of a cell: larger q wins, then the lower slot index.
+__device__ __forceinline__ unsigned long long cell_key(float q, int n) {
+  return ((unsigned long long)ordered_key(q) << 32) | (0xFFFFFFFFu - (uint32_t)n);
+}
+
+// Steps 3-4 over the ordered keys of q~ (keys[0 .. NV) in shared memory).
+// 3. exact K-th largest key by a 4-pass, 8-bit radix select: one histogram
+//    per pass (three buffers in rotation, so a pass needs a single barrier),
+//    and every warp scans the histogram itself to find the digit;
+// 4. ascending emission: each thread owns a contiguous run of slots; one
+//    block-wide exclusive scan of (count above the threshold, count equal to
+//    it), packed in 16-bit halves, gives every kept slot its position.  Among
+//    slots equal to the threshold the lowest indices are kept.
+// Every thread of the block must call it; NV <= 8192.
+static __device__ void select_rank_emit(const uint32_t* keys, int NV, int K, SelectSmem& ss,
+                                        int32_t* keep) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int Kc = min(K, NV);
+  const bool keep_all = Kc == NV;
+  uint32_t thr = 0, need_eq = 0;
+  if (!keep_all && Kc > 0) {
+    for (int i = threadIdx.x; i < 2 * 256; i += blockDim.x) (&ss.hist[0][0])[i] = 0u;
+    __syncthreads();
+    uint32_t prefix = 0, mask = 0, remaining = (uint32_t)Kc;
+    for (int pass = 0; pass < 4; ++pass) {
+      const int shift = 24 - 8 * pass;
+      uint32_t* hist = ss.hist[pass % 3];
+      for (int n = threadIdx.x; n < NV; n += blockDim.x) {
+        const uint32_t k = keys[n];
+        if ((k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1u);
+      }
+      __syncthreads();
+      // the buffer of two passes ahead was last read before this barrier
+      if (pass + 2 < 4)
+        for (int i = threadIdx.x; i < 256; i += blockDim.x) ss.hist[(pass + 2) % 3][i] = 0u;
+      // digit holding the remaining-th largest key, buckets from 255 down
+      uint32_t c[8], tot = 0;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        c[i] = hist[255 - 8 * lane - i];
+        tot += c[i];
+      }
+      uint32_t incl = tot;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      uint32_t excl = incl - tot, digit = 0, rem = 0;
+      const bool here = excl < remaining && remaining <= incl;
+      if (here) {
+        for (int i = 0; i < 8; ++i) {
+          if (excl + c[i] >= remaining) {
+            digit = (uint32_t)(255 - 8 * lane - i);
+            rem = remaining - excl;
+            break;
+          }
+          excl += c[i];
+        }
+      }
+      const int src = __ffs(__ballot_sync(0xffffffffu, here)) - 1;
+      prefix |= __shfl_sync(0xffffffffu, digit, src) << shift;
+      remaining = __shfl_sync(0xffffffffu, rem, src);
+      mask |= 255u << shift;
+    }
+    thr = prefix;
+    need_eq = remaining;
+  }
+
+  // 4. emit ascending indices
+  if (keep_all) {
+    for (int n = threadIdx.x; n < NV; n += blockDim.x) keep[n] = n;
+  } else if (Kc > 0) {
+    const int per = (NV + (int)blockDim.x - 1) / (int)blockDim.x;
+    const int lo = min(NV, (int)threadIdx.x * per), hi = min(NV, lo + per);
+    uint32_t cnt = 0;   // (above threshold) | (equal to it) << 16
+    for (int n = lo; n < hi; ++n) {
+      const uint32_t k = keys[n];
+      cnt += (k > thr) ? 1u : (k == thr ? 0x10000u : 0u);
+    }
+    uint32_t incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (lane == 31) ss.warp_tot[warp] = incl;
+    __syncthreads();
+    uint32_t before = incl - cnt;
+    for (int w = 0; w < warp; ++w) before += ss.warp_tot[w];
+    uint32_t gt = before & 0xFFFFu, eq = before >> 16;
+    for (int n = lo; n < hi; ++n) {
+      const uint32_t k = keys[n];
+      if (k > thr) {
+        keep[gt + min(eq, need_eq)] = n;
+        ++gt;
+      } else if (k == thr) {
+        if (eq < need_eq) keep[gt + eq] = n;
+        ++eq;
+      }
+    }
+  }
+  for (int s = Kc + threadIdx.x; s < K; s += blockDim.x) keep[s] = -1;
+}
+
+// Whole-CTA select for one image.  q[n], cand[n] (nullable) and q_tilde[n]
+// (nullable) are indexed by the image-local slot n in [0, NV); keys (NV
+// words) and cells (NV bytes) are shared scratch; keep receives K entries
+// (ascending, -1 padded).
+static __device__ void select_image(const float* q, const int32_t* cand, int NV, int gh, int gw,
+                                    int G, float lam, int K, uint32_t* keys, uint8_t* cells,
+                                    SelectSmem& ss, float* q_tilde, int32_t* keep,
+                                    uint32_t* status) {
+  const int ncell = G * G;
+  // 1. cell representatives (Eqs. 20-21)
+  for (int i = threadIdx.x; i < ncell; i += blockDim.x) ss.cell_best[i] = 0ull;
+  __syncthreads();
+  for (int n = threadIdx.x; n < NV; n += blockDim.x) {
+    const int g = token_cell(cand, n, gh, gw, G, status);
+    cells[n] = (uint8_t)g;
+    atomicMax(&ss.cell_best[g], cell_key(q[n], n));
+  }
+  __syncthreads();
+  // 2. q~ (Eq. 22)
+  for (int n = threadIdx.x; n < NV; n += blockDim.x) {
+    const uint32_t best = (uint32_t)(ss.cell_best[cells[n]] & 0xFFFFFFFFull);
+    const float bind = (best == 0xFFFFFFFFu - (uint32_t)n) ? 1.f : 0.f;
+    const float qt = (1.f - lam) * q[n] + lam * bind;
+    keys[n] = ordered_key(qt);
+    if (q_tilde) q_tilde[n] = qt;
+  }
+  __syncthreads();
+  // 3-4. threshold of Top-K (Eq. 23) and emission
+  select_rank_emit(keys, NV, K, ss, keep);
+}
+
+// The same select for a CTA that did not compute q: the cell arg-max keys
+// (Eqs. 20-21) were reduced into cell_best_g[0 .. G*G) in global memory by the
+// CTAs that did, and q[] was written by them.  This CTA reads the keys (and
+// resets them to zero for the next use) in the same phase as q, then runs
+// steps 2-4.  keys (NV words) and cells (NV bytes) are shared scratch.
+static __device__ void select_image_from_cells(const float* q, const int32_t* cand, int NV,
+                                               int gh, int gw, int G, float lam, int K,
+                                               unsigned long long* cell_best_g, uint32_t* keys,
+                                               uint8_t* cells, SelectSmem& ss, float* q_tilde,
+                                               int32_t* keep, uint32_t* status) {
+  for (int i = threadIdx.x; i < G * G; i += blockDim.x) {
+    ss.cell_best[i] = __ldcg(cell_best_g + i);
+    cell_best_g[i] = 0ull;
+  }
+  for (int n = threadIdx.x; n < NV; n += blockDim.x) {
+    keys[n] = __float_as_uint(__ldcg(q + n));
+    cells[n] = (uint8_t)token_cell(cand, n, gh, gw, G, status);
+  }
+  __syncthreads();
+  // 2. q~ (Eq. 22)
+  for (int n = threadIdx.x; n < NV; n += blockDim.x) {
+    const uint32_t best = (uint32_t)(ss.cell_best[cells[n]] & 0xFFFFFFFFull);
+    const float bind = (best == 0xFFFFFFFFu - (uint32_t)n) ? 1.f : 0.f;
+    const float qt = (1.f - lam) * __uint_as_float(keys[n]) + lam * bind;
+    keys[n] = ordered_key(qt);
+    if (q_tilde) q_tilde[n] = qt;
+  }
+  __syncthreads();
+  select_rank_emit(keys, NV, K, ss, keep);
+}
+
+// Device-side checks of one image's select arguments.
+__device__ __forceinline__ bool select_args_ok(const LayoutArgs& la, int b, bool has_cand,
+                                               const int32_t* keep_count, const int32_t* keep_off,
+                                               int32_t sum_keep) {
+  const int NV = __ldg(la.n_vis + b), v0 = __ldg(la.vis_off + b);
+  const int gh = __ldg(la.grid_h + b), gw = __ldg(la.grid_w + b);
+  const int K = __ldg(keep_count + b), ko = __ldg(keep_off + b);
+  return NV >= 0 && NV <= la.max_vis && v0 >= 0 && v0 + NV <= la.sum_vis &&
+         __ldg(la.vis_off + b + 1) - v0 == NV && gh > 0 && gw > 0 &&
+         (has_cand ? (long long)gh * gw >= NV : (long long)gh * gw == NV) && K >= 0 && ko >= 0 &&
+         __ldg(keep_off + b + 1) - ko == K && ko + K <= sum_keep;
+}
+
+}  // namespace e2s

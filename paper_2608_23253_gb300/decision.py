@@ -7,6 +7,9 @@ runs in libe2s.so kernels:
     fuse   -> mass, fused (I,U,Theta,K), q (Sec. 4.1-4.2, Eqs. 8-19)
     select -> q~, keep_idx                (Sec. 4.3, Eqs. 20-23)
     compact-> shortened hidden / K / V    (the next layer's input)
+
+decide() runs score, fuse and select through e2s_decide (two launches);
+prune() adds the compaction (e2s_prune, three launches).
 """
 from __future__ import annotations
 
@@ -107,6 +110,14 @@ class Decision:
         e2s.check(e2s.e2s_fuse(self.batch.layout, self.params, self.a, cand, prior, self.mass,
                                self.fused, self.q, self.ws, self.ws_bytes, stream), "e2s_fuse")
 
+    def fuse_select(self, prior: Optional[torch.Tensor] = None,
+                    cand: Optional[torch.Tensor] = None, stream=None) -> None:
+        """fuse + select in one launch (same results as the two calls)."""
+        e2s.check(e2s.e2s_fuse_select(self.batch.layout, self.params, self.a, cand, prior,
+                                      self.mass, self.fused, self.q, self.keep_count,
+                                      self.keep_off, self.sum_keep, self.keep_idx, self.q_tilde,
+                                      self.ws, self.ws_bytes, stream), "e2s_fuse_select")
+
     def select(self, cand: Optional[torch.Tensor] = None, stream=None) -> None:
         e2s.check(e2s.e2s_select(self.batch.layout, self.params, self.q, cand, self.keep_count,
                                  self.keep_off, self.sum_keep, self.keep_idx, self.q_tilde,
@@ -122,11 +133,34 @@ class Decision:
                                   len(src), src, dst, row_bytes, pos_ids, self.ws, self.ws_bytes,
                                   stream), "e2s_compact")
 
+    def decide(self, q_text: torch.Tensor, k: torch.Tensor, prior: Optional[torch.Tensor] = None,
+               cand: Optional[torch.Tensor] = None, stream=None,
+               q_row_stride: Optional[int] = None, k_row_stride: Optional[int] = None) -> None:
+        """score + fuse + select in two launches (e2s_decide)."""
+        b = self.batch
+        qs = q_row_stride if q_row_stride is not None else b.H * b.d
+        ks = k_row_stride if k_row_stride is not None else b.H_kv * b.d
+        e2s.check(e2s.e2s_decide(b.layout, self.params, q_text, qs, k, ks, cand, prior, self.a,
+                                 self.mass, self.fused, self.q, self.keep_count, self.keep_off,
+                                 self.sum_keep, self.keep_idx, self.q_tilde, self.ws,
+                                 self.ws_bytes, stream), "e2s_decide")
+
+    def prune(self, q_text: torch.Tensor, k: torch.Tensor, src: Sequence[torch.Tensor],
+              dst: Sequence[torch.Tensor], pos_ids: Optional[torch.Tensor] = None,
+              prior: Optional[torch.Tensor] = None, cand: Optional[torch.Tensor] = None,
+              stream=None) -> None:
+        """The whole pruning step (e2s_prune): decide, then compact src into dst."""
+        b = self.batch
+        row_bytes = [t.stride(0) * t.element_size() for t in src]
+        e2s.check(e2s.e2s_prune(b.layout, self.params, q_text, b.H * b.d, k, b.H_kv * b.d, cand,
+                                prior, self.a, self.mass, self.fused, self.q, self.keep_count,
+                                self.keep_off, self.sum_keep, self.keep_idx, self.q_tilde,
+                                len(src), src, dst, row_bytes, pos_ids, self.ws, self.ws_bytes,
+                                stream), "e2s_prune")
+
     def run(self, q_text: torch.Tensor, k: torch.Tensor, stream=None) -> None:
-        """score + fuse + select (the decision itself)."""
-        self.score(q_text, k, stream)
-        self.fuse(stream=stream)
-        self.select(stream=stream)
+        """The decision itself: score + fuse + select (e2s_decide)."""
+        self.decide(q_text, k, stream=stream)
 
     def status(self, stream=None) -> int:
         return e2s.e2s_read_status(self.ws, stream)

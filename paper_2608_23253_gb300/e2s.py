@@ -73,7 +73,14 @@ _sz = ctypes.c_size_t
 _SIGS = {
     "e2s_workspace_size": (_sz, [_LP, _PP]),
     "e2s_score": (ctypes.c_int, [_LP, _PP, _vp, _i64, _vp, _i64, _vp, _vp, _sz, _vp]),
+    "e2s_decide": (ctypes.c_int, [_LP, _PP, _vp, _i64, _vp, _i64, _vp, _vp, _vp, _vp, _vp, _vp,
+                                   _vp, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
+    "e2s_prune": (ctypes.c_int, [_LP, _PP, _vp, _i64, _vp, _i64, _vp, _vp, _vp, _vp, _vp, _vp,
+                                  _vp, _vp, _i32, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _sz,
+                                  _vp]),
     "e2s_fuse": (ctypes.c_int, [_LP, _PP, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "e2s_fuse_select": (ctypes.c_int, [_LP, _PP, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _i32,
+                                        _vp, _vp, _vp, _sz, _vp]),
     "e2s_fuse_noalloc": (ctypes.c_int, [_LP, _PP, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
     "e2s_select": (ctypes.c_int, [_LP, _PP, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
     "e2s_compact": (ctypes.c_int, [_LP, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
@@ -126,11 +133,50 @@ def e2s_score(layout, params_, q_text, q_row_stride, k, k_row_stride, a_out, ws,
                          k_row_stride, _ptr(a_out), _ptr(ws), ws_bytes, _stream(stream))
 
 
+def e2s_decide(layout, params_, q_text, q_row_stride, k, k_row_stride, cand, prior, a_out,
+               mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx, q_tilde_out,
+               ws, ws_bytes, stream=None) -> int:
+    return lib.e2s_decide(_ref(layout), _ref(params_), _ptr(q_text), q_row_stride, _ptr(k),
+                          k_row_stride, _ptr(cand), _ptr(prior), _ptr(a_out), _ptr(mass_out),
+                          _ptr(fused_out), _ptr(q_out), _ptr(keep_count), _ptr(keep_off),
+                          sum_keep, _ptr(keep_idx), _ptr(q_tilde_out), _ptr(ws), ws_bytes,
+                          _stream(stream))
+
+
+def _addr_arrays(src, dst, row_bytes, n):
+    src_a = (ctypes.c_void_p * max(n, 1))(*[_ptr(x) for x in src])
+    dst_a = (ctypes.c_void_p * max(n, 1))(*[_ptr(x) for x in dst])
+    rb_a = (ctypes.c_int64 * max(n, 1))(*[int(x) for x in row_bytes])
+    return (ctypes.cast(src_a, ctypes.c_void_p), ctypes.cast(dst_a, ctypes.c_void_p),
+            ctypes.cast(rb_a, ctypes.c_void_p), (src_a, dst_a, rb_a))
+
+
+def e2s_prune(layout, params_, q_text, q_row_stride, k, k_row_stride, cand, prior, a_out,
+              mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx, q_tilde_out,
+              n_tensors, src, dst, row_bytes, pos_ids_out, ws, ws_bytes, stream=None) -> int:
+    """src/dst: sequences of tensors or addresses; row_bytes: sequence of ints."""
+    n = int(n_tensors)
+    s_p, d_p, r_p, _keep = _addr_arrays(src, dst, row_bytes, n)
+    return lib.e2s_prune(_ref(layout), _ref(params_), _ptr(q_text), q_row_stride, _ptr(k),
+                         k_row_stride, _ptr(cand), _ptr(prior), _ptr(a_out), _ptr(mass_out),
+                         _ptr(fused_out), _ptr(q_out), _ptr(keep_count), _ptr(keep_off),
+                         sum_keep, _ptr(keep_idx), _ptr(q_tilde_out), n, s_p, d_p, r_p,
+                         _ptr(pos_ids_out), _ptr(ws), ws_bytes, _stream(stream))
+
+
 def e2s_fuse(layout, params_, a, cand, prior, mass_out, fused_out, q_out, ws, ws_bytes,
              stream=None) -> int:
     return lib.e2s_fuse(_ref(layout), _ref(params_), _ptr(a), _ptr(cand), _ptr(prior),
                         _ptr(mass_out), _ptr(fused_out), _ptr(q_out), _ptr(ws), ws_bytes,
                         _stream(stream))
+
+
+def e2s_fuse_select(layout, params_, a, cand, prior, mass_out, fused_out, q_out, keep_count,
+                    keep_off, sum_keep, keep_idx, q_tilde_out, ws, ws_bytes, stream=None) -> int:
+    return lib.e2s_fuse_select(_ref(layout), _ref(params_), _ptr(a), _ptr(cand), _ptr(prior),
+                               _ptr(mass_out), _ptr(fused_out), _ptr(q_out), _ptr(keep_count),
+                               _ptr(keep_off), sum_keep, _ptr(keep_idx), _ptr(q_tilde_out),
+                               _ptr(ws), ws_bytes, _stream(stream))
 
 
 def e2s_fuse_noalloc(layout, params_, a, cand, prior, mass_out, fused_out, q_out,
@@ -151,13 +197,9 @@ def e2s_compact(layout, keep_idx, keep_off, sum_keep, n_tensors, src, dst, row_b
                 ws, ws_bytes, stream=None) -> int:
     """src/dst: sequences of tensors or addresses; row_bytes: sequence of ints."""
     n = int(n_tensors)
-    src_a = (ctypes.c_void_p * max(n, 1))(*[_ptr(x) for x in src])
-    dst_a = (ctypes.c_void_p * max(n, 1))(*[_ptr(x) for x in dst])
-    rb_a = (ctypes.c_int64 * max(n, 1))(*[int(x) for x in row_bytes])
-    return lib.e2s_compact(_ref(layout), _ptr(keep_idx), _ptr(keep_off), sum_keep, n,
-                           ctypes.cast(src_a, ctypes.c_void_p), ctypes.cast(dst_a, ctypes.c_void_p),
-                           ctypes.cast(rb_a, ctypes.c_void_p), _ptr(pos_ids_out), _ptr(ws),
-                           ws_bytes, _stream(stream))
+    s_p, d_p, r_p, _keep = _addr_arrays(src, dst, row_bytes, n)
+    return lib.e2s_compact(_ref(layout), _ptr(keep_idx), _ptr(keep_off), sum_keep, n, s_p, d_p,
+                           r_p, _ptr(pos_ids_out), _ptr(ws), ws_bytes, _stream(stream))
 
 
 def e2s_read_status(ws, stream=None) -> int:

@@ -211,6 +211,9 @@ def make_inputs(spec: Spec, *, with_payload: bool = True) -> Inputs:
     amp = SIGMA * np.sqrt(d)
     for b, im in enumerate(spec.images):
         rng = np.random.Generator(np.random.PCG64(1000 * spec.cfg_id + b))
+        # V and the hidden states come from a stream of their own, so Q and K
+        # are the same with or without the payload
+        prng = np.random.Generator(np.random.PCG64(1000 * spec.cfg_id + b + (1 << 40)))
         sal = _salient_positions(rng, im.grid_h, im.grid_w, im.n_salient, im.blobs)
         salient.append(sal)
         t0, t1 = int(tok_off[b]), int(tok_off[b + 1])
@@ -227,9 +230,9 @@ def make_inputs(spec: Spec, *, with_payload: bool = True) -> Inputs:
             k[l, t0:t1] = bf16_bits(kk)
             q[l, x0:x1] = bf16_bits(qq)
             if payload:
-                v[l, t0:t1] = bf16_bits(rng.standard_normal((t1 - t0, Hkv, d), dtype=np.float32))
+                v[l, t0:t1] = bf16_bits(prng.standard_normal((t1 - t0, Hkv, d), dtype=np.float32))
         if payload:
-            hid[t0:t1] = bf16_bits(rng.standard_normal((t1 - t0, spec.hidden), dtype=np.float32))
+            hid[t0:t1] = bf16_bits(prng.standard_normal((t1 - t0, spec.hidden), dtype=np.float32))
     return Inputs(spec, n_sys, n_vis, n_text, grid_h, grid_w, tok_off, vis_off, text_off,
                   keep, keep_off, q, k, v, hid, salient)
 

@@ -18,9 +18,16 @@ def device():
     return torch.device("cuda:0")
 
 
+PATHS = ("decide", "fuse_select", "separate")
+
+
 def run_gpu(inp, mode: str = "causal", *, simt: bool = False, flags: int = 0, lam: float = 0.1,
             G: int = 4, keep=None, norm_mode: int = 0, prior=None, cand=None,
-            grid_h=None, grid_w=None):
+            grid_h=None, grid_w=None, path: str = "decide"):
+    """The decision through one of the ABI call sequences:
+    decide       e2s_decide (score, then token-parallel evidence + select)
+    fuse_select  e2s_score, then e2s_fuse_select (one cluster per image)
+    separate     e2s_score, e2s_fuse, e2s_select"""
     from paper_2608_23253_gb300 import e2s
     from paper_2608_23253_gb300.decision import Batch, Decision, bf16_tensor
     dev = device()
@@ -38,9 +45,17 @@ def run_gpu(inp, mode: str = "causal", *, simt: bool = False, flags: int = 0, la
         device=dev)
     cd = None if cand is None else torch.as_tensor(np.concatenate(cand).astype(np.int32),
                                                    device=dev)
-    dec.score(q, k)
-    dec.fuse(prior=pr)
-    dec.select(cand=cd)
+    if path == "decide":
+        dec.decide(q, k, prior=pr, cand=cd)
+    elif path == "fuse_select":
+        dec.score(q, k)
+        dec.fuse_select(prior=pr, cand=cd)
+    elif path == "separate":
+        dec.score(q, k)
+        dec.fuse(prior=pr)
+        dec.select(cand=cd)
+    else:
+        raise ValueError(path)
     torch.cuda.synchronize()
     st = dec.status()
     out = {

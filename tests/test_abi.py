@@ -54,7 +54,8 @@ def test_workspace_size_and_versions():
     e2s = _lib()
     lay = _layout(e2s)
     n = e2s.e2s_workspace_size(lay, e2s.params())
-    assert n == 256 + ((1 * 2 * 32 * 8 + 255) // 256) * 256
+    # status word, one float4 per (image, layer, head), 64 cell keys + a counter per image
+    assert n == 256 + ((1 * 2 * 32 * 16 + 255) // 256) * 256 + ((1 * 129 * 4 + 255) // 256) * 256
     assert e2s.e2s_workspace_size(_layout(e2s, d=64), e2s.params()) == 0
     assert e2s.e2s_version() == 100
     assert e2s.e2s_status_string(e2s.E2S_ERR_TIMEOUT) == "E2S_ERR_TIMEOUT"
@@ -151,3 +152,35 @@ def test_select_and_fuse_host_validation():
     assert e2s.e2s_fuse(lay, par, 0x1000, None, 0x1004, None, 0x1000, 0x2000, ws,
                         1 << 20) == e2s.E2S_ERR_ALIGNMENT
     assert e2s.e2s_read_status(None) == e2s.E2S_ERR_WORKSPACE
+
+
+@pytest.mark.parametrize("case,want", [
+    ("no_keep_count", "E2S_ERR_INVALID_ARG"),
+    ("no_keep_idx", "E2S_ERR_INVALID_ARG"),
+    ("no_a_out", "E2S_ERR_INVALID_ARG"),
+    ("misaligned_fused", "E2S_ERR_ALIGNMENT"),
+    ("small_ws", "E2S_ERR_WORKSPACE"),
+    ("too_many_heads", "E2S_ERR_UNSUPPORTED"),
+])
+def test_decide_host_validation(case, want):
+    e2s = _lib()
+    lay = _layout(e2s)
+    par = e2s.params()
+    ws, wsb = 0x100000, 1 << 20
+    a, fused, keep_count, keep_idx = 0x400000, 0x500000, 0x600000, 0x700000
+    if case == "no_keep_count":
+        keep_count = None
+    elif case == "no_keep_idx":
+        keep_idx = None
+    elif case == "no_a_out":
+        a = None
+    elif case == "misaligned_fused":
+        fused = 0x500008
+    elif case == "small_ws":
+        wsb = e2s.e2s_workspace_size(lay, par) - 4
+    elif case == "too_many_heads":
+        lay = _layout(e2s, H=512, H_kv=512)
+    st = e2s.e2s_decide(lay, par, 0x200000, lay.H * 128, 0x300000, lay.H_kv * 128, None, None,
+                        a, None, fused, 0x580000, keep_count, 0x680000, 64, keep_idx, None,
+                        ws, wsb, None)
+    assert e2s.e2s_status_string(st) == want

@@ -1,0 +1,181 @@
+"""Edge cases, ablation flags, progressive-step arguments and device-side checks (GPU)."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import e2s_oracle as orc
+from paper_2608_23253_gb300 import synth
+from paper_2608_23253_gb300.synth import ImageSpec
+from tests import parity
+from tests.gpu_helpers import PATHS, config_inputs, device, run_gpu, run_oracle
+
+pytestmark = pytest.mark.gpu
+
+ORC_FLAGS = {1: orc.NO_RELIABILITY, 2: orc.NO_LAYER_FUSION, 4: orc.NO_CONFLICT,
+             8: orc.NO_NOVELTY, 16: orc.VANILLA}
+
+
+def _check(inp, gpu, ref, *, lam=0.1, G=4, keep=None, cand=None, grid_h=None, grid_w=None,
+           exact_keep=False):
+    assert gpu["status"] == 0, gpu["status"]
+    parity.check_floats(gpu, ref)
+    parity.check_selection(gpu["keep"], gpu["q_tilde"], ref["q"], inp.n_vis,
+                           inp.grid_h if grid_h is None else grid_h,
+                           inp.grid_w if grid_w is None else grid_w,
+                           inp.keep if keep is None else keep, lam, G, cand=cand)
+    if exact_keep:
+        for b in range(len(inp.n_vis)):
+            assert np.array_equal(gpu["keep"][b], ref["keep"][b])
+
+
+def _spec(images, **kw):
+    return synth.custom_spec("edge", images, **kw)
+
+
+@pytest.mark.parametrize("path", PATHS)
+@pytest.mark.parametrize("mode", ["causal", "eq1"])
+def test_ragged_extremes(mode, path):
+    """1x1 and non-divisible grids, N_T = 1, K = 0 and K > N_V in one ragged batch."""
+    ims = [ImageSpec(35, 1, 1, 1, 1, 0, 1), ImageSpec(3, 5, 7, 17, 4, 0, 0),
+           ImageSpec(35, 36, 36, 128, 90, 3, 144), ImageSpec(0, 9, 13, 2, 10, 2, 200),
+           ImageSpec(35, 24, 24, 64, 40, 3, 64)]
+    inp = synth.make_inputs(_spec(ims, L=3, H=8, H_kv=8, cfg_id=90), with_payload=False)
+    gpu = run_gpu(inp, mode, path=path)
+    ref = run_oracle(inp, mode)
+    _check(inp, gpu, ref)
+    assert gpu["keep"][1].size == 0
+    assert gpu["keep"][3].tolist() == list(range(117)) + [-1] * 83
+
+
+@pytest.mark.parametrize("mode", ["causal", "eq1"])
+def test_max_text_rows(mode):
+    ims = [ImageSpec(35, 16, 16, 256, 20, 3, 28), ImageSpec(35, 24, 24, 200, 30, 3, 64)]
+    inp = synth.make_inputs(_spec(ims, L=2, H=4, H_kv=4, cfg_id=91), with_payload=False)
+    _check(inp, run_gpu(inp, mode), run_oracle(inp, mode))
+
+
+@pytest.mark.parametrize("mode", ["causal", "eq1"])
+def test_gqa_split_head_groups(mode):
+    """Group of 7 query heads with 128 text rows: the heads of a kv head are split over CTAs."""
+    ims = [ImageSpec(35, 16, 16, 128, 20, 3, 28), ImageSpec(35, 24, 32, 100, 50, 3, 85)]
+    inp = synth.make_inputs(_spec(ims, L=2, H=14, H_kv=2, cfg_id=92), with_payload=False)
+    _check(inp, run_gpu(inp, mode), run_oracle(inp, mode))
+
+
+def test_all_equal_scores_tie_break():
+    """Zero queries give equal logits everywhere: ties resolve to the lower index."""
+    inp = config_inputs(0, None, None)
+    import copy
+    inp = copy.copy(inp)
+    inp.q_text = np.zeros_like(inp.q_text)
+    gpu = run_gpu(inp, "causal")
+    ref = run_oracle(inp, "causal")
+    _check(inp, gpu, ref, exact_keep=True)
+    gpu = run_gpu(inp, "eq1")
+    ref = run_oracle(inp, "eq1")
+    _check(inp, gpu, ref, exact_keep=True)
+
+
+@pytest.mark.parametrize("flag", [1, 2, 4, 8, 16])
+def test_ablation_flags(flag):
+    inp = config_inputs(1, None, None)
+    gpu = run_gpu(inp, "causal", flags=flag)
+    ref = run_oracle(inp, "causal", flags=ORC_FLAGS[flag])
+    lam = 0.0 if flag in (8, 16) else 0.1
+    _check(inp, gpu, ref, lam=lam)
+
+
+@pytest.mark.parametrize("norm", ["softmax", "renorm"])
+def test_norm_modes_causal(norm):
+    inp = config_inputs(0, None, None)
+    nm = {"softmax": 1, "renorm": 2}[norm]
+    gpu = run_gpu(inp, "causal", norm_mode=nm)
+    ref = run_oracle(inp, "causal", norm=norm)
+    _check(inp, gpu, ref)
+
+
+@pytest.mark.parametrize("G,lam", [(1, 0.1), (3, 0.3), (8, 0.05)])
+def test_cell_counts_and_lambda(G, lam):
+    inp = config_inputs(1, None, None)
+    _check(inp, run_gpu(inp, "causal", G=G, lam=lam), run_oracle(inp, "causal", G=G, lam=lam),
+           lam=lam, G=G)
+
+
+@pytest.mark.parametrize("path", PATHS)
+def test_progressive_prior_and_candidates(path):
+    """A later pruning step: 122 surviving candidates of a 24 x 24 grid, fused state carried."""
+    r = np.random.default_rng(7)
+    cand = [np.sort(r.choice(576, size=122, replace=False)),
+            np.sort(r.choice(576, size=48, replace=False))]
+    ims = [ImageSpec(35, 1, 122, 64, 0, 0, 48), ImageSpec(35, 1, 48, 30, 0, 0, 42)]
+    inp = synth.make_inputs(_spec(ims, L=2, H=32, H_kv=32, cfg_id=93), with_payload=False)
+    gh, gw = np.array([24, 24]), np.array([24, 24])
+    prior = r.dirichlet([1.0, 1.0, 1.0], size=int(inp.n_vis.sum()))
+    gpu = run_gpu(inp, "causal", prior=prior, cand=cand, grid_h=gh, grid_w=gw, path=path)
+    ref = run_oracle(inp, "causal", prior=prior, cand=cand, grid_h=gh, grid_w=gw)
+    _check(inp, gpu, ref, cand=cand, grid_h=gh, grid_w=gw)
+
+
+def test_padded_row_strides():
+    from paper_2608_23253_gb300 import e2s
+    from paper_2608_23253_gb300.decision import Batch, Decision, bf16_tensor
+    dev = device()
+    inp = config_inputs(0, None, None)
+    s = inp.spec
+    L, St, Sx = s.L, int(inp.tok_off[-1]), int(inp.text_off[-1])
+    qpad = np.zeros((L, Sx, s.H * 128 + 64), dtype=np.uint16)
+    qpad[:, :, :s.H * 128] = inp.q_text.reshape(L, Sx, -1)
+    kpad = np.zeros((L, St, s.H_kv * 128 + 8), dtype=np.uint16)
+    kpad[:, :, :s.H_kv * 128] = inp.k.reshape(L, St, -1)
+    batch = Batch.from_inputs(inp, device=dev)
+    dec = Decision(batch, inp.keep, e2s.params())
+    dec.score(bf16_tensor(qpad, dev), bf16_tensor(kpad, dev), q_row_stride=qpad.shape[2],
+              k_row_stride=kpad.shape[2])
+    torch.cuda.synchronize()
+    assert dec.status() == 0
+    ref = run_oracle(inp, "causal")
+    parity.assert_close("a", dec.a.cpu().numpy(), ref["a"])
+
+
+@pytest.mark.parametrize("decide", [False, True])
+def test_device_detects_inconsistent_layout(decide):
+    """A layout whose device arrays disagree is reported through the status word."""
+    from paper_2608_23253_gb300 import e2s
+    from paper_2608_23253_gb300.decision import Batch, Decision, bf16_tensor
+    dev = device()
+    inp = config_inputs(0, None, None)
+    batch = Batch.from_inputs(inp, device=dev)
+    batch.array("n_vis")[0] += 1          # no longer matches vis_off / tok_off / the grid
+    dec = Decision(batch, inp.keep, e2s.params())
+    if decide:
+        dec.decide(bf16_tensor(inp.q_text, dev), bf16_tensor(inp.k, dev))
+    else:
+        dec.score(bf16_tensor(inp.q_text, dev), bf16_tensor(inp.k, dev))
+        dec.fuse_select()
+    torch.cuda.synchronize()
+    assert dec.status() == e2s.E2S_ERR_SHAPE
+    assert e2s.e2s_clear_status(dec.ws) == e2s.E2S_OK
+    assert dec.status() == e2s.E2S_OK
+
+
+def test_deterministic_repeat():
+    inp = config_inputs(2, 4, None)
+    g1 = run_gpu(inp, "causal")
+    g2 = run_gpu(inp, "causal")
+    for key in ("a", "mass", "fused", "q", "q_tilde"):
+        assert np.array_equal(g1[key], g2[key]), key
+    for b in range(4):
+        assert np.array_equal(g1["keep"][b], g2["keep"][b])
+
+
+@pytest.mark.parametrize("path", ["fuse_select", "separate"])
+def test_call_sequences_agree(path):
+    """e2s_decide against the other two call sequences on one ragged GQA batch."""
+    inp = config_inputs(3, 4, None)
+    g1 = run_gpu(inp, "causal", path="decide")
+    g2 = run_gpu(inp, "causal", path=path)
+    assert np.array_equal(g1["a"], g2["a"])
+    for key in ("mass", "fused", "q", "q_tilde"):
+        parity.assert_close(key, g1[key], g2[key], tol=1e-5)
+    for b in range(4):
+        assert np.array_equal(g1["keep"][b], g2["keep"][b])

@@ -24,7 +24,7 @@ def _id(c):
 
 
 @pytest.mark.parametrize("mode", ["causal", "eq1"])
-@pytest.mark.parametrize("path", ["tc", "simt"])
+@pytest.mark.parametrize("path", ["decide", "fuse_select", "simt"])
 @pytest.mark.parametrize("case", CASES, ids=_id)
 def test_decision_parity(case, path, mode):
     cfg, batch, keep = case
@@ -32,7 +32,12 @@ def test_decision_parity(case, path, mode):
         pytest.skip("keep budget does not affect the score kernel")
     inp = config_inputs(cfg, batch, keep)
     ref = config_oracle(cfg, batch, keep, mode)
-    gpu = run_gpu(inp, mode, simt=(path == "simt"))
+    # decide: e2s_decide on the tensor-core score; fuse_select: tensor-core
+    # e2s_score, then the cluster launch; simt: SIMT e2s_score, then the
+    # separate e2s_fuse and e2s_select calls
+    gpu = run_gpu(inp, mode, simt=(path == "simt"),
+                  path={"decide": "decide", "fuse_select": "fuse_select",
+                        "simt": "separate"}[path])
     assert gpu["status"] == 0, gpu["status"]
     parity.check_floats(gpu, ref)
     parity.check_selection(gpu["keep"], gpu["q_tilde"], ref["q"], inp.n_vis, inp.grid_h,
@@ -94,3 +99,41 @@ def test_ragged_compaction_bit_exact():
     assert np.array_equal(out.cpu().view(torch.int16).numpy().view(np.uint16), want)
     assert np.array_equal(pos.cpu().numpy(),
                           orc.position_ids(inp.n_sys, inp.n_vis, inp.n_text, ref["keep"]))
+
+
+@pytest.mark.parametrize("cfg,batch", [(1, None), (2, 6), (3, 4)], ids=["cfg1", "cfg2-b6",
+                                                                        "cfg3-b4"])
+def test_prune_whole_step(cfg, batch):
+    """e2s_prune (decide, then compaction whose fixed rows overlap the decision):
+    the decision matches the oracle, and every output row is the oracle's
+    compaction of the keep set the GPU chose, bit for bit."""
+    from paper_2608_23253_gb300 import e2s
+    from paper_2608_23253_gb300.decision import Batch, Decision, bf16_tensor
+    dev = device()
+    inp = config_inputs(cfg, batch, None, True)
+    ref = config_oracle(cfg, batch, None, "causal")
+    dec = Decision(Batch.from_inputs(inp, device=dev), inp.keep, e2s.params())
+    L = inp.spec.L
+    host = [inp.hidden] + [inp.k[l].reshape(inp.k.shape[1], -1) for l in range(L)] + \
+           [inp.v[l].reshape(inp.v.shape[1], -1) for l in range(L)]
+    src = [bf16_tensor(x, dev) for x in host]
+    R = dec.out_rows()
+    dst = [torch.full((R, t.shape[1]), -1, dtype=t.dtype, device=dev) for t in src]
+    pos = torch.full((R,), -7, dtype=torch.int32, device=dev)
+    dec.prune(bf16_tensor(inp.q_text, dev), bf16_tensor(inp.k, dev), src, dst, pos)
+    torch.cuda.synchronize()
+    assert dec.status() == 0
+    gpu = {"a": dec.a.cpu().numpy(), "mass": dec.mass.cpu().numpy(),
+           "fused": dec.fused.cpu().numpy(), "q": dec.q.cpu().numpy(),
+           "q_tilde": dec.q_tilde.cpu().numpy(), "keep": dec.keep_lists()}
+    parity.check_floats(gpu, ref)
+    parity.check_selection(gpu["keep"], gpu["q_tilde"], ref["q"], inp.n_vis, inp.grid_h,
+                           inp.grid_w, inp.keep, 0.1, 4)
+    if parity.oracle_keep_ok(ref, inp.n_vis, inp.keep):
+        for b in range(inp.spec.B):
+            assert np.array_equal(gpu["keep"][b], ref["keep"][b])
+    for d_, h_ in zip(dst, host):
+        want = orc.compact(h_, inp.n_sys, inp.n_vis, inp.n_text, gpu["keep"])
+        assert np.array_equal(d_.cpu().view(torch.int16).numpy().view(np.uint16), want)
+    assert np.array_equal(pos.cpu().numpy(),
+                          orc.position_ids(inp.n_sys, inp.n_vis, inp.n_text, gpu["keep"]))

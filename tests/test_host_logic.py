@@ -65,6 +65,17 @@ def test_generator_deterministic_and_planted():
     assert norms[sal].mean() > 3 * norms[others].mean()
 
 
+def test_payload_does_not_change_q_and_k():
+    """V and the hidden states come from their own stream: a test that needs the
+    payload may reuse the oracle computed on the inputs without it."""
+    spec = synth.config_spec(0)
+    spec.hidden = 64
+    a = synth.make_inputs(spec, with_payload=True)
+    b = synth.make_inputs(spec, with_payload=False)
+    assert np.array_equal(a.k, b.k) and np.array_equal(a.q_text, b.q_text)
+    assert a.v is not None and b.v is None and a.hidden.shape == (643, 64)
+
+
 def test_blobs_are_spatially_clustered():
     spec = synth.config_spec(1)
     inp = synth.make_inputs(spec, with_payload=False)
