@@ -130,13 +130,13 @@ e2s_status e2s_score(const e2s_layout* layout, const e2s_params* params,
  * a_out is required (it carries a[l][h][n] from the first launch to the
  * second).  The score kernel also leaves the Eq. 8 normalisation statistics
  * of every (image, layer, head) in the workspace, so the second kernel treats
- * every visual token independently (64 tokens per CTA) and the last CTA to
+ * every visual token independently (one warp per token) and the last CTA to
  * finish an image runs that image's Top-K.  Results are identical to
  * e2s_score, e2s_fuse and e2s_select called in sequence, up to the rounding
  * order of the normalisation sums.  keep_count and keep_off are required;
  * keep_idx may be NULL only when sum_keep == 0.  Concurrent e2s_decide calls
- * must use separate workspaces.  E2S_ERR_UNSUPPORTED when H > 384 or
- * L * H > 4096. */
+ * must use separate workspaces.  E2S_ERR_UNSUPPORTED when H > 128 or when
+ * L * H * 84 + 5 * max_vis bytes exceed 160 KiB (L * H > 1900 or so). */
 e2s_status e2s_decide(const e2s_layout* layout, const e2s_params* params,
                       const void* q_text, int64_t q_row_stride,
                       const void* k, int64_t k_row_stride,

@@ -7,12 +7,14 @@
 #include <algorithm>
 
 #include "device_common.cuh"
+#include "sm100_ptx.cuh"
 
 namespace e2s {
 namespace {
 
 constexpr int kCompactThreads = 256;
 constexpr int kRowVec = 16;   // 16-byte vectors per lane in flight
+constexpr long long kPrefetchBytes = 48ll << 20;   // candidate rows prefetched into L2
 
 struct TensorSet {
   const char* src[kMaxCompactTensors];
@@ -93,17 +95,36 @@ __device__ __forceinline__ void compact_rows(const LayoutArgs& la, const int32_t
   }
 }
 
+// L2 prefetch of every candidate visual row of every tensor (one bulk
+// prefetch per row), so that the rows the selection keeps are L2 hits.
+__device__ __forceinline__ void prefetch_visual_rows(const LayoutArgs& la, int n_tensors,
+                                                     const TensorSet& ts) {
+  const long long total = (long long)la.sum_vis * n_tensors;
+  for (long long pr = (long long)blockIdx.x * blockDim.x + threadIdx.x; pr < total;
+       pr += (long long)gridDim.x * blockDim.x) {
+    const int tix = (int)(pr / la.sum_vis);
+    const int gv = (int)(pr - (long long)tix * la.sum_vis);
+    const int b = find_segment(la.vis_off, la.B, gv);
+    const long long row = (long long)__ldg(la.tok_off + b) + __ldg(la.n_sys + b) +
+                          (gv - __ldg(la.vis_off + b));
+    if (row < 0 || row >= la.sum_T) continue;   // inconsistent layout: the copy flags it
+    ptx::prefetch_l2_bulk(ts.src[tix] + row * ts.row_bytes[tix], (uint32_t)ts.row_bytes[tix]);
+  }
+}
+
 // early != 0: the system and text rows (which do not depend on the selection)
 // are copied before griddepcontrol.wait, overlapping the kernel that writes
 // keep_idx; the caller guarantees that the sources and keep_off were complete
-// before that kernel's predecessor started.
+// before that kernel's predecessor started.  prefetch != 0 (with early): the
+// candidate visual rows are also prefetched into L2 while waiting.
 __global__ void __launch_bounds__(kCompactThreads)
     compact_kernel(const LayoutArgs la, const int32_t* __restrict__ keep_idx,
                    const int32_t* __restrict__ keep_off, int n_tensors, const TensorSet ts,
                    int32_t* __restrict__ pos_ids, long long total_rows, uint32_t* status,
-                   int early) {
+                   int early, int prefetch) {
   pdl_launch_dependents();
   if (early) {
+    if (prefetch) prefetch_visual_rows(la, n_tensors, ts);
     compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, 0);
     pdl_wait();   // keep_idx comes from the previous kernel
     compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, 1);
@@ -127,13 +148,23 @@ cudaError_t launch_compact(const LayoutArgs& la, const int32_t* keep_idx, const 
     ts.dst[i] = static_cast<char*>(dst[i]);
     ts.row_bytes[i] = row_bytes[i];
   }
+  // prefetching every candidate row pays while those rows fit comfortably
+  // in L2 (a single image or a small batch); larger batches are bandwidth-bound
+  long long row_sum = 0;
+  bool rows_small = true;
+  for (int i = 0; i < n_tensors; ++i) {
+    row_sum += row_bytes[i];
+    rows_small = rows_small && row_bytes[i] <= (1ll << 20);
+  }
+  const int prefetch =
+      early && rows_small && (long long)la.sum_vis * row_sum <= kPrefetchBytes ? 1 : 0;
   const long long pairs = total_rows * (n_tensors > 0 ? n_tensors : 1);
   const int warps_per_block = kCompactThreads / 32;
   long long blocks = (pairs + warps_per_block - 1) / warps_per_block;
   blocks = std::min<long long>(blocks, (long long)sm_count() * 16);
   return launch_kernel(compact_kernel, dim3((unsigned)std::max<long long>(blocks, 1)),
                        dim3(kCompactThreads), 0, st, 0, true, la, keep_idx, keep_off, n_tensors, ts,
-                       pos_ids, total_rows, status, early);
+                       pos_ids, total_rows, status, early, prefetch);
 }
 
 }  // namespace e2s

@@ -1,21 +1,22 @@
 // Evidence, layer-wise fusion and selection of e2s_decide (Sec. 4.1-4.3,
 // Eqs. 8-23), token-parallel.  The normalisation statistics of Eq. 8 for
 // every (image, layer, head) were produced by the score kernel, so tokens are
-// independent here: a CTA takes 64 visual tokens of one image, eight lanes per
-// token (one eighth of the heads each):
+// independent here.  A CTA of 256 threads takes 64 visual tokens of one image:
 //   1. the image's statistics and the CTA's a[l][h][token] values are copied
-//      into shared memory with asynchronous copies (16-byte copies when the
-//      rows are aligned), all of a group of layers in flight at once;
-//   2. per (token, layer): supports p (Eq. 9) of the lane's heads, kept in
-//      registers; p_bar and the reliability terms of Eq. 10 summed over the
-//      eight lanes with three shuffles; rho and the layer mass (Eq. 11);
-//   3. per token: Dempster combination over the layers (Eqs. 12-16), Pl and q
-//      (Eqs. 18-19);
-//   4. every CTA folds its tokens' bids for their cells' representatives
-//      (Eqs. 20-21) into the image's cell arg-max keys in global memory and
-//      bumps the image's arrival counter; the last CTA of the image computes
-//      q~ and the Top-K (Eqs. 22-23) over the whole image and re-arms the
-//      keys and the counter.
+//      into shared memory with asynchronous copies, all in flight at once;
+//   2. one thread per (token, layer) walks the H heads: supports p (Eq. 9),
+//      written back over the staged scores, p_bar, then the reliability terms
+//      of Eq. 10, rho and the layer mass (Eq. 11) -- independent iterations,
+//      no cross-thread reduction;
+//   3. one thread per token: Dempster combination of its layer masses in
+//      order (Eqs. 12-16), Pl and q (Eqs. 18-19), and its bid for its cell's
+//      representative (Eqs. 20-21);
+//   4. every CTA folds its bids into the image's cell arg-max keys in global
+//      memory and bumps the image's arrival counter; the last CTA of the image
+//      computes q~ and the Top-K (Eqs. 22-23) over the whole image and re-arms
+//      the keys and the counter.
+// The select arguments are inputs of the call, not results of the score
+// kernel, so they are checked before griddepcontrol.wait.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -26,12 +27,20 @@
 namespace e2s {
 namespace {
 
-constexpr int kTok = 64;                 // visual tokens per CTA
-constexpr int kLanes = 8;                // lanes per token (head groups)
-constexpr int kDecThreads = kLanes * kTok;
-constexpr int kMaxHpl = 8;               // supports cached per lane (H <= 64)
+constexpr int kTok = 64;                           // visual tokens per CTA
+constexpr int kRow = kTok;                         // staged row stride (floats)
+constexpr int kDecThreads = 256;
+constexpr int kLayerLanes = kDecThreads / kTok;    // layers handled side by side
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr size_t kDecStageBytes = 96u << 10;   // staged scores per group of layers
+constexpr size_t kDecSmemBudget = 160u << 10;
+
+// [L][H] statistics, [L][kTok] layer masses and head sums, then the staged
+// scores [L][H][kRow] (reused as the select's keys and cell ids).
+__host__ __device__ inline size_t dec_smem_bytes(int L, int H, int max_vis) {
+  const size_t st = (size_t)L * H * 16 + (size_t)L * kTok * 20;
+  const size_t a = (size_t)L * H * kRow * 4;
+  return st + std::max(a, (size_t)max_vis * 5);
+}
 
 struct DecArgs {
   LayoutArgs la;
@@ -40,7 +49,6 @@ struct DecArgs {
   float lam;
   int G;
   int blocks_per_image;
-  int lps;   // evidence layers staged at a time
   const float* a;
   const float4* stats;
   const float4* prior;
@@ -70,13 +78,6 @@ __device__ __forceinline__ float support_p(float a, float4 st, int softmax, floa
   return x * fast_rcp(1.f + x);                     // Eq. 9
 }
 
-__device__ __forceinline__ float lane_sum8(float v) {
-  v += __shfl_xor_sync(0xffffffffu, v, 1);
-  v += __shfl_xor_sync(0xffffffffu, v, 2);
-  v += __shfl_xor_sync(0xffffffffu, v, 4);
-  return v;
-}
-
 __global__ void __launch_bounds__(kDecThreads) decide_kernel(const DecArgs p) {
   extern __shared__ __align__(16) uint8_t dec_smem[];
   __shared__ SelectSmem ss;
@@ -84,13 +85,12 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const DecArgs p) {
   __shared__ unsigned long long cb_s[kDecideCells];   // this CTA's cell arg-max keys
   const LayoutArgs& la = p.la;
   const int H = la.H, L = la.L;
-  // [L][H] statistics, then [lps][H][kTok] staged scores (the select's scratch later)
-  float4* st_s = reinterpret_cast<float4*>(dec_smem);
-  float* A = reinterpret_cast<float*>(dec_smem + (size_t)L * H * 16);
+  float4* st_s = reinterpret_cast<float4*>(dec_smem);           // [L][H]
+  float4* M_s = st_s + (size_t)L * H;                            // [L][kTok]
+  float* SA_s = reinterpret_cast<float*>(M_s + (size_t)L * kTok);  // [L][kTok]
+  float* A = SA_s + (size_t)L * kTok;                            // [L][H][kRow]
   const int tid = threadIdx.x;
   for (int i = tid; i < kDecideCells; i += kDecThreads) cb_s[i] = 0ull;
-  pdl_launch_dependents();
-  pdl_wait();   // a and the statistics come from the score kernel
 
   const int b = blockIdx.x / p.blocks_per_image;
   const int blk = blockIdx.x - b * p.blocks_per_image;
@@ -100,156 +100,127 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const DecArgs p) {
   const int n0 = blk * kTok;
   const int ntok = ok ? max(0, min(kTok, NV - n0)) : 0;
   const size_t plane = (size_t)la.sum_vis;
-  // 16-byte copies need every staged row segment 16-byte aligned
-  const bool vec = ((reinterpret_cast<uintptr_t>(p.a) | ((plane & 3) << 2) |
-                     ((size_t)(v0 + n0) << 2)) & 15) == 0;
-
-  // the image's statistics (every layer) arrive with the first group of scores
-  for (int i = tid; i < L * H * 4; i += kDecThreads)
-    ptx::cp_async4(reinterpret_cast<float*>(st_s) + i,
-                   reinterpret_cast<const float*>(p.stats + (size_t)b * L * H) + i);
-
-  // 2-3. evidence and fusion, lanes 8j .. 8j+7 own token j
-  const int j = tid / kLanes, hq = tid % kLanes;
-  const bool live = j < ntok;
-  const int gv = v0 + n0 + j;
-  const float N = (float)NV;
-  const float invN = NV > 0 ? 1.f / N : 0.f;
-  const float inv_h = 1.f / (float)H;
-  const int hpl = (H + kLanes - 1) / kLanes;
-  const int h_lo = hq * hpl, h_cnt = max(0, min(H, h_lo + hpl) - h_lo);
-  float fI = 0.f, fU = 0.f, fT = 1.f, K = 0.f, vsum = 0.f;
-  bool have = false;
-  if (live && p.prior != nullptr && !(p.flags & E2S_NO_LAYER_FUSION)) {
-    const float4 pr = p.prior[gv];
-    fI = pr.x; fU = pr.y; fT = pr.z;
-    have = true;
-  }
-  const int l_begin = (p.flags & E2S_NO_LAYER_FUSION) ? L - 1 : 0;
-  for (int l = 0; l < L; ++l) {
-    const int li = l % p.lps;
-    if (li == 0) {
-      // 1. stage a[l .. l+lps)[h][n0 .. n0+ntok) (coalesced along the tokens)
-      const int nl = min(p.lps, L - l);
-      __syncthreads();   // the previous group is consumed
-      if (vec) {
-        for (int idx = tid; idx < nl * H * (kTok / 4); idx += kDecThreads) {
-          const int jj = 4 * (idx & (kTok / 4 - 1)), lh = idx / (kTok / 4);
-          const float* src = p.a + ((size_t)l * H + lh) * plane + v0 + n0 + jj;
-          if (jj + 4 <= ntok) {
-            ptx::cp_async16(A + lh * kTok + jj, src);
-          } else {
-            for (int e = 0; e < 4; ++e)
-              if (jj + e < ntok) ptx::cp_async4(A + lh * kTok + jj + e, src + e);
-          }
-        }
-      } else {
-        for (int idx = tid; idx < nl * H * kTok; idx += kDecThreads) {
-          const int jj = idx & (kTok - 1), lh = idx / kTok;
-          if (jj < ntok)
-            ptx::cp_async4(A + idx, p.a + ((size_t)l * H + lh) * plane + v0 + n0 + jj);
-        }
-      }
-      ptx::cp_async_wait_all();
-      __syncthreads();
-    }
-    const float* Al = A + (size_t)li * H * kTok + j;
-    const float4* sl = st_s + (size_t)l * H;
-    float pv[kMaxHpl];
-    float sum_p = 0.f, sum_a = 0.f;
-#pragma unroll
-    for (int k = 0; k < kMaxHpl; ++k) {
-      pv[k] = 0.f;
-      if (live && k < h_cnt) {
-        const int h = h_lo + k;
-        const float av = Al[h * kTok];
-        sum_a += av;
-        pv[k] = support_p(av, sl[h], p.softmax, N, invN);
-        sum_p += pv[k];
-      }
-    }
-    if (live)
-      for (int h = h_lo + kMaxHpl; h < h_lo + h_cnt; ++h) {   // H > 64 only
-        const float av = Al[h * kTok];
-        sum_a += av;
-        sum_p += support_p(av, sl[h], p.softmax, N, invN);
-      }
-    sum_p = lane_sum8(sum_p);
-    sum_a = lane_sum8(sum_a);
-    const float p_bar = sum_p * inv_h;
-    float clar = 0.f, dev = 0.f;
-#pragma unroll
-    for (int k = 0; k < kMaxHpl; ++k)
-      if (live && k < h_cnt) {
-        clar += pv[k] - 0.5f;
-        dev += fabsf(pv[k] - p_bar);
-      }
-    if (live)
-      for (int h = h_lo + kMaxHpl; h < h_lo + h_cnt; ++h) {
-        const float v = support_p(Al[h * kTok], sl[h], p.softmax, N, invN);
-        clar += v - 0.5f;
-        dev += fabsf(v - p_bar);
-      }
-    clar = lane_sum8(clar);
-    dev = lane_sum8(dev);
-    float rho = (2.f * inv_h) * fabsf(clar) * (1.f - (2.f * inv_h) * dev);  // Eq. 10
-    if (p.flags & E2S_NO_RELIABILITY) rho = 1.f;
-    const float mI = rho * p_bar, mU = rho * (1.f - p_bar), mT = 1.f - rho;  // Eq. 11
-    if (live && hq == 0 && p.mass_out)
-      p.mass_out[(size_t)l * plane + gv] = make_float4(mI, mU, mT, p_bar);
-    vsum += sum_a;
-    if (l < l_begin) continue;
-    if (!have) {                                   // Eq. 12
-      fI = mI; fU = mU; fT = mT; K = 0.f;
-      have = true;
-    } else {                                       // Eqs. 13-16
-      const float Kc = fI * mU + fU * mI;
-      const float omk = 1.f - Kc;
-      if (omk <= 0.f) {
-        fI = 0.f; fU = 0.f; fT = 1.f; K = 1.f;
-      } else {
-        const float inv = 1.f / omk;
-        const float nI = (fI * mI + fI * mT + fT * mI) * inv;
-        const float nU = (fU * mU + fU * mT + fT * mU) * inv;
-        const float nT = fT * mT * inv;
-        fI = nI; fU = nU; fT = nT; K = Kc;
-      }
-    }
-  }
   const bool select = p.keep_count != nullptr;
   const int G = p.G;
   const int gh = __ldg(la.grid_h + b), gw = __ldg(la.grid_w + b);
-  if (live && hq == 0) {
+  const bool sel_ok =
+      select && ok &&
+      select_args_ok(la, b, p.cand != nullptr, p.keep_count, p.keep_off, p.sum_keep);
+  const CellMap cells(gh, gw, G);
+  pdl_launch_dependents();
+  pdl_wait();   // a and the statistics come from the score kernel
+
+  // 1. stage the statistics and a[l][h][n0 .. n0+ntok) (coalesced along the tokens)
+  for (int i = tid; i < L * H * 4; i += kDecThreads)
+    ptx::cp_async4(reinterpret_cast<float*>(st_s) + i,
+                   reinterpret_cast<const float*>(p.stats + (size_t)b * L * H) + i);
+  for (int idx = tid; idx < L * H * kTok; idx += kDecThreads) {
+    const int jj = idx & (kTok - 1), lh = idx >> 6;
+    if (jj < ntok) ptx::cp_async4(A + lh * kRow + jj, p.a + (size_t)lh * plane + v0 + n0 + jj);
+  }
+  ptx::cp_async_wait_all();
+  __syncthreads();
+
+  // 2. per (token, layer): supports, reliability and layer mass (Eqs. 8-11)
+  const float N = (float)NV;
+  const float invN = NV > 0 ? 1.f / N : 0.f;
+  const float inv_h = 1.f / (float)H;
+  {
+    const int j = tid & (kTok - 1);
+    for (int l = tid / kTok; l < L; l += kLayerLanes) {
+      if (j >= ntok) continue;
+      float* Ac = A + (size_t)l * H * kRow + j;
+      const float4* sl = st_s + (size_t)l * H;
+      float sum_p = 0.f, sum_a = 0.f;
+#pragma unroll 8
+      for (int h = 0; h < H; ++h) {
+        const float av = Ac[h * kRow];
+        const float pv = support_p(av, sl[h], p.softmax, N, invN);
+        sum_a += av;
+        sum_p += pv;
+        Ac[h * kRow] = pv;
+      }
+      const float p_bar = sum_p * inv_h;
+      float clar = 0.f, dev = 0.f;
+#pragma unroll 8
+      for (int h = 0; h < H; ++h) {
+        const float pv = Ac[h * kRow];
+        clar += pv - 0.5f;
+        dev += fabsf(pv - p_bar);
+      }
+      float rho = (2.f * inv_h) * fabsf(clar) * (1.f - (2.f * inv_h) * dev);  // Eq. 10
+      if (p.flags & E2S_NO_RELIABILITY) rho = 1.f;
+      const float4 m4 = make_float4(rho * p_bar, rho * (1.f - p_bar), 1.f - rho, p_bar);  // Eq. 11
+      M_s[l * kTok + j] = m4;
+      SA_s[l * kTok + j] = sum_a;
+      if (p.mass_out) p.mass_out[(size_t)l * plane + v0 + n0 + j] = m4;
+    }
+  }
+  __syncthreads();
+
+  // 3. per token: Dempster combination over the layers (Eqs. 12-16), q (Eq. 19)
+  if (tid < ntok) {
+    const int j = tid, gv = v0 + n0 + j;
+    float fI = 0.f, fU = 0.f, fT = 1.f, K = 0.f, vsum = 0.f;
+    bool have = false;
+    if (p.prior != nullptr && !(p.flags & E2S_NO_LAYER_FUSION)) {
+      const float4 pr = p.prior[gv];
+      fI = pr.x; fU = pr.y; fT = pr.z;
+      have = true;
+    }
+    const int l_begin = (p.flags & E2S_NO_LAYER_FUSION) ? L - 1 : 0;
+    for (int l = 0; l < L; ++l) {
+      vsum += SA_s[l * kTok + j];
+      if (l < l_begin) continue;
+      const float4 m = M_s[l * kTok + j];
+      if (!have) {                                   // Eq. 12
+        fI = m.x; fU = m.y; fT = m.z; K = 0.f;
+        have = true;
+      } else {                                       // Eqs. 13-16
+        const float Kc = fI * m.y + fU * m.x;
+        const float omk = 1.f - Kc;
+        if (omk <= 0.f) {
+          fI = 0.f; fU = 0.f; fT = 1.f; K = 1.f;
+        } else {
+          const float inv = 1.f / omk;
+          const float nI = (fI * m.x + fI * m.z + fT * m.x) * inv;
+          const float nU = (fU * m.y + fU * m.z + fT * m.y) * inv;
+          const float nT = fT * m.z * inv;
+          fI = nI; fU = nU; fT = nT; K = Kc;
+        }
+      }
+    }
     const float Pl = fI + fT;                                                   // Eq. 18
     float q = (p.flags & E2S_NO_CONFLICT) ? Pl : 1.f - (1.f - Pl) * (1.f - K);  // Eq. 19
     if (p.flags & E2S_VANILLA) q = vsum / (float)(L * H);
     p.fused_out[gv] = make_float4(fI, fU, fT, K);
     p.q_out[gv] = q;
-    // 4a. this token's bid for its cell's representative (Eqs. 20-21)
-    const int n = n0 + j;
-    if (select && gh > 0 && gw > 0)
-      atomicMax(&cb_s[token_cell(p.cand ? p.cand + v0 : nullptr, n, gh, gw, G, p.status)],
+    // bid for the cell's representative (Eqs. 20-21)
+    if (sel_ok) {
+      const int n = n0 + j;
+      atomicMax(&cb_s[token_cell(p.cand ? p.cand + v0 : nullptr, n, cells, p.status)],
                 cell_key(q, n));
+    }
   }
   if (!select) return;
   __syncthreads();
   for (int i = tid; i < G * G; i += kDecThreads)
     if (cb_s[i] != 0ull) atomicMax(p.cell_best + (size_t)b * kDecideCells + i, cb_s[i]);
 
-  // 4b. the last CTA of the image selects; the barrier orders every thread's
-  // writes before thread 0's fence and arrival
+  // 4. the last CTA of the image selects.  The barrier orders every thread's
+  // writes before thread 0's acquire-release arrival; in the last CTA the
+  // arrival's acquire plus the barrier after it make every other CTA's
+  // writes visible to all of its threads.
   __syncthreads();
   if (tid == 0) {
-    __threadfence();
-    const uint32_t ticket = atomicAdd(p.counters + b, 1u);
+    const uint32_t ticket = ptx::atom_add_acq_rel_gpu(p.counters + b, 1u);
     is_last = ticket == (uint32_t)(p.blocks_per_image - 1);
+    if (is_last) p.counters[b] = 0u;   // re-armed for the next call
   }
   __syncthreads();
   if (!is_last) return;
-  __threadfence();
-  if (tid == 0) p.counters[b] = 0u;   // re-armed for the next call
   unsigned long long* cells_g = p.cell_best + (size_t)b * kDecideCells;
-  if (!(ok && select_args_ok(la, b, p.cand != nullptr, p.keep_count, p.keep_off, p.sum_keep))) {
+  if (!sel_ok) {
     for (int i = tid; i < kDecideCells; i += kDecThreads) cells_g[i] = 0ull;
     if (tid == 0) E2S_DEV_FLAG(p.status, E2S_ERR_SHAPE);
     return;
@@ -265,7 +236,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const DecArgs p) {
 }  // namespace
 
 bool decide_fits(const LayoutArgs& la) {
-  return (size_t)la.H * kTok * 4 <= kDecStageBytes && (size_t)la.L * la.H * 16 <= (64u << 10);
+  return dec_smem_bytes(la.L, la.H, la.max_vis) <= kDecSmemBudget;
 }
 
 cudaError_t launch_decide(const LayoutArgs& la, int norm_softmax, uint32_t flags, float lambda,
@@ -280,7 +251,6 @@ cudaError_t launch_decide(const LayoutArgs& la, int norm_softmax, uint32_t flags
     *unsupported = 1;
     return cudaSuccess;
   }
-  const size_t layer_bytes = (size_t)la.H * kTok * 4;
   DecArgs p;
   p.la = la;
   p.softmax = norm_softmax;
@@ -288,7 +258,6 @@ cudaError_t launch_decide(const LayoutArgs& la, int norm_softmax, uint32_t flags
   p.lam = lambda;
   p.G = G;
   p.blocks_per_image = (la.max_vis + kTok - 1) / kTok;
-  p.lps = (int)std::min<size_t>((size_t)la.L, kDecStageBytes / layer_bytes);
   p.a = a;
   p.stats = stats;
   p.prior = reinterpret_cast<const float4*>(prior);
@@ -304,8 +273,7 @@ cudaError_t launch_decide(const LayoutArgs& la, int norm_softmax, uint32_t flags
   p.cell_best = reinterpret_cast<unsigned long long*>(scratch);
   p.counters = scratch + (size_t)2 * kDecideCells * la.B;
   p.status = status;
-  const size_t smem =
-      (size_t)la.L * la.H * 16 + std::max((size_t)p.lps * layer_bytes, (size_t)la.max_vis * 5);
+  const size_t smem = dec_smem_bytes(la.L, la.H, la.max_vis);
   return launch_kernel(decide_kernel, dim3((unsigned)(la.B * p.blocks_per_image)),
                        dim3(kDecThreads), smem, st, 0, true, p);
 }

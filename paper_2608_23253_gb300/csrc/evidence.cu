@@ -331,6 +331,7 @@ cudaError_t launch_evidence(const LayoutArgs& la, int norm_softmax, uint32_t fla
     *unsupported = 1;
     return cudaSuccess;
   }
+  p.ts = std::max(p.ts, 2);   // the multiplier of a stride of 1 does not fit 32 bits
   int dev = 0, optin = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;

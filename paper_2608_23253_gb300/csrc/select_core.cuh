@@ -22,7 +22,19 @@ struct SelectSmem {
   unsigned long long cell_best[kMaxCells];
   uint32_t hist[3][256];   // one per radix pass, rotating (zeroed two passes ahead)
   uint32_t warp_tot[32];
+  uint32_t w_and[32], w_or[32];   // per warp AND / OR of the keys
 };
+
+// Per-warp AND and OR of the keys a thread wrote (identity values for none);
+// the whole block calls it before the barrier that publishes the keys.
+__device__ __forceinline__ void publish_key_bits(uint32_t k_and, uint32_t k_or, SelectSmem& ss) {
+  k_and = __reduce_and_sync(0xffffffffu, k_and);
+  k_or = __reduce_or_sync(0xffffffffu, k_or);
+  if ((threadIdx.x & 31) == 0) {
+    ss.w_and[threadIdx.x >> 5] = k_and;
+    ss.w_or[threadIdx.x >> 5] = k_or;
+  }
+}
 
 // Exclusive prefix count of `flag` over the block (in thread order) and the
 // block total.  Every thread of the block must call it.
@@ -49,17 +61,43 @@ __device__ __forceinline__ int cell_id(int r, int gh, int gw, int G) {
   return (i * G / gh) * G + (j * G / gw);
 }
 
+// n / d for 0 <= n < 2^17 and 2 <= d <= 2^13 as a multiply-high with
+// m = ceil(2^32 / d): the product exceeds n/d by less than n / 2^32 < 2^-15,
+// while a non-integer n/d is at least 1/d >= 2^-13 below the next integer,
+// so the floor is exact.  (The multiplier of d = 1 does not fit 32 bits.)
+__device__ __forceinline__ uint32_t div_multiplier(int d) {
+  return d >= 2 ? (uint32_t)((0x100000000ull + (uint64_t)d - 1) / (uint64_t)d) : 0u;
+}
+
+// The G x G cell grid of one image: cell(i, j) = (i*G/h, j*G/w) of raster
+// index r = i*w + j, with multiply-high divisions where they are exact.
+struct CellMap {
+  int gh, gw, G;
+  uint32_t m_gh, m_gw;
+  bool fast;
+  __device__ __forceinline__ CellMap(int gh_, int gw_, int G_) : gh(gh_), gw(gw_), G(G_) {
+    fast = gh >= 2 && gw >= 2 && gh <= 8192 && gw <= 8192 && (long long)gh * gw < (1 << 17);
+    m_gh = fast ? div_multiplier(gh) : 0u;
+    m_gw = fast ? div_multiplier(gw) : 0u;
+  }
+  __device__ __forceinline__ int operator()(int r) const {
+    if (!fast) return cell_id(r, gh, gw, G);
+    const int i = (int)__umulhi((uint32_t)r, m_gw), j = r - i * gw;
+    return (int)__umulhi((uint32_t)(i * G), m_gh) * G + (int)__umulhi((uint32_t)(j * G), m_gw);
+  }
+};
+
 // Cell of image-local slot n: its original raster index (cand, when given)
-// mapped to the G x G grid of cells.  An out-of-range candidate raises
-// E2S_ERR_SHAPE and is clamped.
-__device__ __forceinline__ int token_cell(const int32_t* cand, int n, int gh, int gw, int G,
+// mapped to the cell grid.  An out-of-range candidate raises E2S_ERR_SHAPE and
+// is clamped.
+__device__ __forceinline__ int token_cell(const int32_t* cand, int n, const CellMap& cm,
                                           uint32_t* status) {
   int r = cand ? __ldg(cand + n) : n;
-  if (r < 0 || r >= gh * gw) {
+  if (r < 0 || r >= cm.gh * cm.gw) {
     E2S_DEV_FLAG(status, E2S_ERR_SHAPE);
-    r = min(max(r, 0), gh * gw - 1);
+    r = min(max(r, 0), cm.gh * cm.gw - 1);
   }
-  return cell_id(r, gh, gw, G);
+  return cm(r);
 }
 
 // Arg-max key of a cell: larger q wins, then the lower slot index.
@@ -70,7 +108,9 @@ __device__ __forceinline__ unsigned long long cell_key(float q, int n) {
 // Steps 3-4 over the ordered keys of q~ (keys[0 .. NV) in shared memory).
 // 3. exact K-th largest key by a 4-pass, 8-bit radix select: one histogram
 //    per pass (three buffers in rotation, so a pass needs a single barrier),
-//    and every warp scans the histogram itself to find the digit;
+//    and every warp scans the histogram itself to find the digit; a pass
+//    whose 8 bits are the same in every key (from the AND / OR of all keys
+//    that publish_key_bits left in ss) is skipped;
 // 4. ascending emission: each thread owns a contiguous run of slots; one
 //    block-wide exclusive scan of (count above the threshold, count equal to
 //    it), packed in 16-bit halves, gives every kept slot its position.  Among
@@ -83,20 +123,32 @@ static __device__ void select_rank_emit(const uint32_t* keys, int NV, int K, Sel
   const bool keep_all = Kc == NV;
   uint32_t thr = 0, need_eq = 0;
   if (!keep_all && Kc > 0) {
+    uint32_t all_and = 0xFFFFFFFFu, all_or = 0u;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+      all_and &= ss.w_and[w];
+      all_or |= ss.w_or[w];
+    }
+    const uint32_t same = ~(all_and ^ all_or);   // bits equal in every key
     for (int i = threadIdx.x; i < 2 * 256; i += blockDim.x) (&ss.hist[0][0])[i] = 0u;
     __syncthreads();
     uint32_t prefix = 0, mask = 0, remaining = (uint32_t)Kc;
+    int ex = 0;   // executed passes: executed pass e uses buffer e % 3
     for (int pass = 0; pass < 4; ++pass) {
       const int shift = 24 - 8 * pass;
-      uint32_t* hist = ss.hist[pass % 3];
+      if (((same >> shift) & 255u) == 255u) {   // every key has this digit
+        prefix |= all_and & (255u << shift);
+        mask |= 255u << shift;
+        continue;
+      }
+      uint32_t* hist = ss.hist[ex % 3];
       for (int n = threadIdx.x; n < NV; n += blockDim.x) {
         const uint32_t k = keys[n];
         if ((k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1u);
       }
       __syncthreads();
-      // the buffer of two passes ahead was last read before this barrier
-      if (pass + 2 < 4)
-        for (int i = threadIdx.x; i < 256; i += blockDim.x) ss.hist[(pass + 2) % 3][i] = 0u;
+      // the buffer of two executed passes ahead was last read before this barrier
+      for (int i = threadIdx.x; i < 256; i += blockDim.x) ss.hist[(ex + 2) % 3][i] = 0u;
+      ++ex;
       // digit holding the remaining-th largest key, buckets from 255 down
       uint32_t c[8], tot = 0;
 #pragma unroll
@@ -176,23 +228,29 @@ static __device__ void select_image(const float* q, const int32_t* cand, int NV,
                                     SelectSmem& ss, float* q_tilde, int32_t* keep,
                                     uint32_t* status) {
   const int ncell = G * G;
+  const CellMap cm(gh, gw, G);
   // 1. cell representatives (Eqs. 20-21)
   for (int i = threadIdx.x; i < ncell; i += blockDim.x) ss.cell_best[i] = 0ull;
   __syncthreads();
   for (int n = threadIdx.x; n < NV; n += blockDim.x) {
-    const int g = token_cell(cand, n, gh, gw, G, status);
+    const int g = token_cell(cand, n, cm, status);
     cells[n] = (uint8_t)g;
     atomicMax(&ss.cell_best[g], cell_key(q[n], n));
   }
   __syncthreads();
   // 2. q~ (Eq. 22)
+  uint32_t k_and = 0xFFFFFFFFu, k_or = 0u;
   for (int n = threadIdx.x; n < NV; n += blockDim.x) {
     const uint32_t best = (uint32_t)(ss.cell_best[cells[n]] & 0xFFFFFFFFull);
     const float bind = (best == 0xFFFFFFFFu - (uint32_t)n) ? 1.f : 0.f;
     const float qt = (1.f - lam) * q[n] + lam * bind;
-    keys[n] = ordered_key(qt);
+    const uint32_t k = ordered_key(qt);
+    keys[n] = k;
+    k_and &= k;
+    k_or |= k;
     if (q_tilde) q_tilde[n] = qt;
   }
+  publish_key_bits(k_and, k_or, ss);
   __syncthreads();
   // 3-4. threshold of Top-K (Eq. 23) and emission
   select_rank_emit(keys, NV, K, ss, keep);
@@ -208,23 +266,29 @@ static __device__ void select_image_from_cells(const float* q, const int32_t* ca
                                                unsigned long long* cell_best_g, uint32_t* keys,
                                                uint8_t* cells, SelectSmem& ss, float* q_tilde,
                                                int32_t* keep, uint32_t* status) {
+  const CellMap cm(gh, gw, G);
   for (int i = threadIdx.x; i < G * G; i += blockDim.x) {
     ss.cell_best[i] = __ldcg(cell_best_g + i);
     cell_best_g[i] = 0ull;
   }
   for (int n = threadIdx.x; n < NV; n += blockDim.x) {
     keys[n] = __float_as_uint(__ldcg(q + n));
-    cells[n] = (uint8_t)token_cell(cand, n, gh, gw, G, status);
+    cells[n] = (uint8_t)token_cell(cand, n, cm, status);
   }
   __syncthreads();
   // 2. q~ (Eq. 22)
+  uint32_t k_and = 0xFFFFFFFFu, k_or = 0u;
   for (int n = threadIdx.x; n < NV; n += blockDim.x) {
     const uint32_t best = (uint32_t)(ss.cell_best[cells[n]] & 0xFFFFFFFFull);
     const float bind = (best == 0xFFFFFFFFu - (uint32_t)n) ? 1.f : 0.f;
     const float qt = (1.f - lam) * __uint_as_float(keys[n]) + lam * bind;
-    keys[n] = ordered_key(qt);
+    const uint32_t k = ordered_key(qt);
+    keys[n] = k;
+    k_and &= k;
+    k_or |= k;
     if (q_tilde) q_tilde[n] = qt;
   }
+  publish_key_bits(k_and, k_or, ss);
   __syncthreads();
   select_rank_emit(keys, NV, K, ss, keep);
 }

@@ -97,6 +97,25 @@ __device__ __forceinline__ void cp_async4(void* dst_smem, const void* src_gmem) 
                "l"(src_gmem)
                : "memory");
 }
+// Device-scope fetch-and-add with acquire-release semantics: the thread's
+// earlier writes (and those ordered before it by a CTA barrier) are visible
+// to whoever observes the new value, and writes released before the value it
+// reads are visible to this thread afterwards.
+__device__ __forceinline__ uint32_t atom_add_acq_rel_gpu(uint32_t* addr, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;"
+               : "=r"(old)
+               : "l"(addr), "r"(v)
+               : "memory");
+  return old;
+}
+
+// Bulk prefetch of [src, src + bytes) into L2 (no completion to wait for);
+// src 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void prefetch_l2_bulk(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 // 16-byte asynchronous copy that bypasses L1; both addresses 16-byte aligned.
 __device__ __forceinline__ void cp_async16(void* dst_smem, const void* src_gmem) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst_smem)),

@@ -47,6 +47,17 @@ def test_ragged_extremes(mode, path):
     assert gpu["keep"][3].tolist() == list(range(117)) + [-1] * 83
 
 
+@pytest.mark.parametrize("path", PATHS)
+def test_single_token_images(path):
+    """A batch made only of 1 x 1 grids (every per-image slice is one token long)."""
+    ims = [ImageSpec(35, 1, 1, 7, 1, 0, 1), ImageSpec(2, 1, 1, 1, 0, 0, 0),
+           ImageSpec(0, 1, 1, 3, 0, 0, 2)]
+    inp = synth.make_inputs(_spec(ims, L=2, H=8, H_kv=8, cfg_id=94), with_payload=False)
+    gpu = run_gpu(inp, "causal", path=path)
+    _check(inp, gpu, run_oracle(inp, "causal"))
+    assert [k.tolist() for k in gpu["keep"]] == [[0], [], [0, -1]]
+
+
 @pytest.mark.parametrize("mode", ["causal", "eq1"])
 def test_max_text_rows(mode):
     ims = [ImageSpec(35, 16, 16, 256, 20, 3, 28), ImageSpec(35, 24, 24, 200, 30, 3, 64)]

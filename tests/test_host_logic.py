@@ -84,3 +84,20 @@ def test_blobs_are_spatially_clustered():
     # 40 points in 3 blobs: the mean nearest-neighbour distance is ~1 grid step
     d = np.sqrt((i[:, None] - i[None]) ** 2 + (j[:, None] - j[None]) ** 2) + np.eye(s.size) * 99
     assert d.min(axis=1).mean() < 1.5
+
+
+def test_multiply_high_division_is_exact():
+    """The cell arithmetic of the select divides small non-negative ints by 2 <= d <= 2^13 as
+    umulhi(n, ceil(2^32 / d)) (d = 1 takes a plain division: its multiplier
+    does not fit 32 bits); the claim is exactness for every n < 2^17.
+    Checked at the worst numerators n = q*d + d - 1 (largest fractional part)
+    and at the multiples n = q*d, for every d."""
+    import numpy as np
+    for d in range(2, 8193):
+        assert ((1 << 32) + d - 1) // d < (1 << 32)
+        m = ((1 << 32) + d - 1) // d
+        q = np.arange(0, (1 << 17) // d + 1, dtype=np.uint64)
+        for n in (q * np.uint64(d), q * np.uint64(d) + np.uint64(d - 1)):
+            n = n[n < (1 << 17)]
+            got = (n * np.uint64(m)) >> np.uint64(32)
+            assert np.array_equal(got, n // np.uint64(d)), d
