@@ -50,14 +50,74 @@ WORKLOADS = {
                             "4 layers, 32x128 MHA, K=11% (configs[4])"),
 }
 
-# ncu dram__bytes_read.sum + dram__bytes_write.sum of one score-kernel launch on this
-# workload, and the sha256 (first 16 hex) of csrc/score_tc.cu when it was captured.
-NCU_TRAFFIC = {"score_tc_kernel": None}
+# ncu dram__bytes_read.sum + dram__bytes_write.sum of one launch of the dominant
+# kernel on a workload (ncu --set full, its default cache control: cold caches),
+# with the sha256 (first 16 hex) of the kernel's source when it was captured; a
+# source that has changed since reports null traffic.
+NCU_TRAFFIC = {
+    "cfg1": {"stage": "score", "kernel": "score_unit_kernel", "src": "score_unit.cu",
+             "sha": "72f9be68c2e4f653", "bytes": 18223104 + 256},
+}
 
 
 def _src_hash(name: str) -> str:
     p = os.path.join(ROOT, "paper_2608_23253_gb300", "csrc", name)
     return hashlib.sha256(open(p, "rb").read()).hexdigest()[:16]
+
+
+def combine_ranks(total_ms: float, e2e_ms: float, images_per_rank: int, world: int, device):
+    """Whole-job numbers of a replicas run: the MAX over ranks of the timed
+    totals (every rank times the same number of steps) and the rate of all the
+    images every rank processed over that time."""
+    import torch
+    t = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    total, e2e = float(t[0]), float(t[1])
+    images = images_per_rank * world
+    return total, e2e, images / (total * 1e-3), images / (e2e * 1e-3)
+
+
+def layer_prefill_us(seq: int, dev, reps: int = 20) -> float:
+    """Comparator only (torch, not this library): one LLaMA-2-7B / LLaVA-1.5-7B
+    decoder layer's prefill at `seq` tokens -- RMSNorm, fused QKV projection,
+    causal attention (bf16 matmuls, fp32 softmax), output projection, RMSNorm,
+    SwiGLU MLP (4096 -> 11008) -- in bf16 with random weights; mean of `reps`
+    CUDA-event-timed runs after warm-up."""
+    import torch
+    import torch.nn.functional as F
+    g = torch.Generator(device=dev).manual_seed(7)
+    D, Hh, I = 4096, 32, 11008
+    w = lambda *sh: (torch.randn(*sh, device=dev, generator=g, dtype=torch.bfloat16) * 0.02)  # noqa: E731
+    wqkv, wo, wgu, wd = w(3 * D, D), w(D, D), w(2 * I, D), w(D, I)
+    x = torch.randn(seq, D, device=dev, generator=g, dtype=torch.bfloat16)
+
+    def rms(v):
+        return v * torch.rsqrt(v.float().pow(2).mean(-1, keepdim=True) + 1e-6).to(v.dtype)
+
+    causal = torch.full((seq, seq), float("-inf"), device=dev).triu(1)
+    scale = (D // Hh) ** -0.5
+
+    def layer(h):
+        qkv = rms(h) @ wqkv.t()
+        q, k, v = qkv.view(seq, 3, Hh, D // Hh).permute(1, 2, 0, 3).contiguous()
+        pr = torch.softmax(torch.matmul(q, k.transpose(1, 2)).float() * scale + causal, -1)
+        o = torch.matmul(pr.to(torch.bfloat16), v)
+        h = h + o.permute(1, 0, 2).reshape(seq, D) @ wo.t()
+        gu = rms(h) @ wgu.t()
+        return h + (F.silu(gu[:, :I]) * gu[:, I:]) @ wd.t()
+
+    for _ in range(3):
+        layer(x)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(reps):
+        layer(x)
+    e1.record()
+    e1.synchronize()
+    return e0.elapsed_time(e1) * 1e3 / reps
 
 
 def measured_peaks():
@@ -329,15 +389,8 @@ def run_ours(args, world, rank, local):
             if it >= args.warmup:
                 e2e_ms.append(e0.elapsed_time(e1))
 
-    total_ms = sum(step_ms)
-    if world > 1:
-        t = torch.tensor([total_ms, sum(e2e_ms)], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms, e2e_total = float(t[0]), float(t[1])
-    else:
-        e2e_total = sum(e2e_ms)
-    images = batch.B * args.steps * world
-    value = images / (total_ms * 1e-3)
+    total_ms, e2e_total, value, e2e_value = combine_ranks(
+        sum(step_ms), sum(e2e_ms), batch.B * args.steps, world, dev)
 
     # roofline of the dominant kernel.  Algorithmic bytes: score reads K of the
     # whole sequence and the text queries once and writes a; the decision
@@ -352,6 +405,7 @@ def run_ours(args, world, rank, local):
         "compact": 2 * R * sum(t.stride(0) * t.element_size() for t in src) + R * 4,
     }
     mean_ms = {n: statistics.mean(v_) for n, v_ in stage_ms.items()}
+    decision_us = mean_ms["decide"] * 1e3   # e2s_decide alone: score + decision kernels
     # e2s_decide is the score kernel plus the decision kernel: the decision
     # kernel's own time is the difference of the two isolated graphs
     mean_ms["decide"] = max(mean_ms["decide"] - mean_ms["score"], 1e-6)
@@ -360,9 +414,9 @@ def run_ours(args, world, rank, local):
     peak, peak_src = (peaks["hbm_gbs"], "measured") if peaks else (6800.0, "fallback")
     achieved = bytes_stage[dom] / (mean_ms[dom] * 1e-3) / 1e9
     traffic = None
-    key = "score_tc_kernel" if dom == "score" else None
-    if key and NCU_TRAFFIC.get(key) and NCU_TRAFFIC[key]["src"] == _src_hash("score_tc.cu"):
-        traffic = NCU_TRAFFIC[key]["bytes"]
+    rec = NCU_TRAFFIC.get(args.workload)
+    if rec and rec["stage"] == dom and rec["sha"] == _src_hash(rec["src"]):
+        traffic = rec["bytes"]
     clk = clocks.summary()
     if rank != 0:
         return
@@ -387,11 +441,26 @@ def run_ours(args, world, rank, local):
                        "frac_hbm": bytes_stage[n] / (mean_ms[n] * 1e-3) / 1e9 / peak}
                    for n in stages},
         "gpu_launches": launches_per_step * args.steps,
-        "e2e": {"value": images / (e2e_total * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "clocks": clk,
         "wall_s_timed_region": t_wall,
     }
+    if world == 1 and args.workload == "cfg1":
+        T = batch.sum_T
+        lay = layer_prefill_us(T, dev)
+        # the layer's dense work: projections and MLP (2 * T * params) plus causal attention
+        flops = 2.0 * T * (4096 * 3 * 4096 + 4096 * 4096 + 3 * 4096 * 11008) \
+            + 2.0 * 2.0 * 4096 * T * (T + 1) / 2.0
+        tf = (peaks or {}).get("bf16_tflops_sustained") or 1700.0
+        est = flops / (tf * 1e12) * 1e6
+        line["decision_vs_layer_prefill"] = {
+            "decision_us": decision_us, "layer_prefill_us": lay, "frac": decision_us / lay,
+            "layer_prefill_est_us": est, "frac_of_est": decision_us / est,
+            "note": "decision = e2s_decide graph (score + evidence/fusion/Top-K), L2 flushed; "
+                    "layer = torch bf16 comparator, one LLaMA-2-7B decoder layer at the same "
+                    "sequence length, random weights; est = its FLOPs at the measured "
+                    "sustained bf16 peak"}
     if world == 1 and not args.no_cpu_baseline:
         rate, info = cpu_oracle_rate(args.workload)
         line["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
