@@ -39,7 +39,8 @@ constexpr size_t kDecSmemBudget = 160u << 10;
 __host__ __device__ inline size_t dec_smem_bytes(int L, int H, int max_vis) {
   const size_t st = (size_t)L * H * 16 + (size_t)L * kTok * 20;
   const size_t a = (size_t)L * H * kRow * 4;
-  return st + std::max(a, (size_t)max_vis * 5);
+  const size_t sel = (size_t)max_vis * 5;
+  return st + (a > sel ? a : sel);
 }
 
 struct DecArgs {

@@ -1,0 +1,434 @@
+// Text-to-visual score, streaming variant for long sequences and grouped-query
+// attention (tcgen05 + TMEM, TMA-streamed bf16 K tiles; Sec. 3.1 Eq. 1 and its
+// causal-prefix probability reading).  Used when a unit's K does not fit in
+// shared memory or its heads share K (GQA), for at most 128 text rows.
+//
+// One CTA per SM loops over units (image, layer, query head); the query head
+// reads kv head h / (H / H_kv).  The MMA is transposed with respect to the
+// persistent single-CTA kernel: D[t][key] = Q[t][:] . K_tile[key][:] with the
+// 128 text rows on the TMEM lanes (M = 128) and 128 keys per tile on the
+// columns (N = 128), so each text row's softmax over its keys is lane-local:
+//   sweep 1 every key tile of the causal prefix (keys 0 .. S+N_V+N_T-1):
+//           each lane keeps a running (max, sum of exp2) of its row over the
+//           32 columns its warp reads -- no cross-lane work; at the end the
+//           four column groups merge into lse_t (log2 domain) per row;
+//   sweep 2 the visual tiles again (the MMAs are recomputed from re-streamed
+//           K): P = exp2(s - lse_t), column sums over the rows (butterfly
+//           reduce-scatter inside a warp, then the four lane quarters in a
+//           fixed order through shared memory), a[key] = sum_t P / N_T.
+// EQ1 mode has no sweep 1 and sums s / sqrt(d) / N_T in sweep 2.
+// K tiles stream through a 4-stage ring (TMA producer warp), the accumulator
+// is double-buffered in TMEM (MMA warp), so loads, MMAs and the epilogue of
+// consecutive tiles overlap.
+//
+// Warp roles (576 threads): warp 0 TMA producer, warp 1 TMEM allocator and MMA
+// issuer, warps 2-17 epilogue: warp w reads TMEM lane quarter w % 4 (text rows
+// 32*(w%4) ..) and column group (w - 2) / 4 (32 keys of each tile).
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+
+#include "sm100_ptx.cuh"
+
+namespace e2s {
+
+bool make_score_map(CUtensorMap* map, const void* base, int heads, int64_t rows,
+                    int64_t row_stride_el, int box_rows);
+
+namespace {
+
+constexpr int kRows = 128;                    // text rows per unit (M)
+constexpr int kTileKeys = 128;                // keys per tile (N)
+constexpr int kHalfBytes = 128 * 128;         // 128 rows x 64 bf16
+constexpr int kTileBytes = 2 * kHalfBytes;    // one 128 x 128 bf16 operand
+constexpr int kStages = 4;
+constexpr int kEpiWarps = 16;
+constexpr int kEpiThreads = 32 * kEpiWarps;
+constexpr int kThreads = 64 + kEpiThreads;
+constexpr uint64_t kWaitNs = 1000000000ull;
+constexpr uint64_t kWaitNsAfterFault = 1000000ull;
+constexpr float kLog2e = 1.4426950408889634f;
+
+struct StreamArgs {
+  LayoutArgs la;
+  int mode;
+  int group;            // query heads per kv head
+  int num_units;
+  float scale;          // 1 / sqrt(d)
+  float scale_log2;     // log2(e) / sqrt(d)
+  float* a_out;
+  float4* stats;        // per (image, layer, head) statistics of the visual scores
+  uint32_t* counters;   // nullable: decision scratch to zero
+  uint32_t* status;
+};
+
+struct SPlan {
+  uint32_t q, k, bars, slot, ms, cps, red, as, total;
+};
+
+__host__ __device__ inline SPlan stream_plan(int max_vis) {
+  SPlan s;
+  s.q = 0;                                              // [2 halves][128 rows][128 B]
+  s.k = (uint32_t)kTileBytes;                           // [kStages][tile]
+  s.bars = s.k + (uint32_t)kStages * kTileBytes;        // 2 + 2*kStages + 4 mbarriers
+  s.slot = s.bars + 8u * (uint32_t)(2 + 2 * kStages + 4);
+  s.ms = (s.slot + 16u + 15u) & ~15u;                   // [4][128] float2 (max, sum)
+  s.cps = s.ms + 4u * kRows * 8u;                       // [2][4][128] column partials
+  s.red = s.cps + 2u * 4u * kTileKeys * 4u;             // [2][kEpiWarps] float2
+  s.as = s.red + 2u * kEpiWarps * 8u;                   // [max_vis] the unit's scores
+  s.total = s.as + (uint32_t)(max_vis > 1 ? max_vis : 1) * 4u;
+  return s;
+}
+
+template <int W, int MASK, class Op>
+__device__ __forceinline__ void rs_step(float (&x)[16], bool hi, Op op) {
+#pragma unroll
+  for (int i = 0; i < W; ++i) {
+    const float send = hi ? x[i] : x[i + W];
+    const float keep = hi ? x[i + W] : x[i];
+    x[i] = op(keep, __shfl_xor_sync(0xffffffffu, send, MASK));
+  }
+}
+// lane L ends with column L >> 1 of the 16, reduced over all 32 lanes
+template <class Op>
+__device__ __forceinline__ float reduce_scatter16(float (&x)[16], int lane, Op op) {
+  rs_step<8, 16>(x, lane & 16, op);
+  rs_step<4, 8>(x, lane & 8, op);
+  rs_step<2, 4>(x, lane & 4, op);
+  rs_step<1, 2>(x, lane & 2, op);
+  return op(x[0], __shfl_xor_sync(0xffffffffu, x[0], 1));
+}
+struct AddOp {
+  __device__ __forceinline__ float operator()(float a, float b) const { return a + b; }
+};
+
+// Geometry of one unit, derived identically by every warp role.
+struct SGeo {
+  int b, l, h, kvh, S, NV, NT, t0, x0, v0;
+  int n1, n2;   // key tiles of sweep 1 (whole causal prefix) and sweep 2 (visual)
+  bool ok;
+};
+
+__device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit) {
+  const LayoutArgs& la = p.la;
+  SGeo g;
+  g.h = unit % la.H;
+  g.l = (unit / la.H) % la.L;
+  g.b = unit / (la.H * la.L);
+  g.kvh = g.h / p.group;
+  g.S = __ldg(la.n_sys + g.b);
+  g.NV = __ldg(la.n_vis + g.b);
+  g.NT = __ldg(la.n_text + g.b);
+  g.t0 = __ldg(la.tok_off + g.b);
+  g.x0 = __ldg(la.text_off + g.b);
+  g.v0 = __ldg(la.vis_off + g.b);
+  const int T = g.S + g.NV + g.NT;
+  g.ok = g.S >= 0 && g.NV >= 0 && g.NT >= 1 && g.NT <= kRows && T <= la.max_T &&
+         g.NV <= la.max_vis && __ldg(la.tok_off + g.b + 1) - g.t0 == T && g.t0 >= 0 &&
+         g.t0 + T <= la.sum_T && __ldg(la.text_off + g.b + 1) - g.x0 == g.NT && g.x0 >= 0 &&
+         g.x0 + g.NT <= la.sum_text && __ldg(la.vis_off + g.b + 1) - g.v0 == g.NV &&
+         g.v0 >= 0 && g.v0 + g.NV <= la.sum_vis;
+  const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
+  g.n1 = g.ok && causal ? (T + kTileKeys - 1) / kTileKeys : 0;
+  g.n2 = g.ok ? (g.NV + kTileKeys - 1) / kTileKeys : 0;
+  return g;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    score_stream_kernel(const __grid_constant__ CUtensorMap tmQ,
+                        const __grid_constant__ CUtensorMap tmK, const StreamArgs p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const LayoutArgs& la = p.la;
+  const SPlan plan = stream_plan(la.max_vis);
+  uint8_t* q_sm = smem + plan.q;
+  uint8_t* k_sm = smem + plan.k;
+  uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + plan.bars);
+  uint64_t* q_empty = q_full + 1;
+  uint64_t* k_full = q_empty + 1;          // [kStages]
+  uint64_t* k_empty = k_full + kStages;    // [kStages]
+  uint64_t* a_full = k_empty + kStages;    // [2] accumulator buffer ready
+  uint64_t* a_empty = a_full + 2;          // [2] accumulator buffer read
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + plan.slot);
+  float2* ms = reinterpret_cast<float2*>(smem + plan.ms);
+  float* cps = reinterpret_cast<float*>(smem + plan.cps);
+  float2* red = reinterpret_cast<float2*>(smem + plan.red);
+  float* as = reinterpret_cast<float*>(smem + plan.as);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
+  pdl_launch_dependents();   // every CTA is resident: the next kernel may be scheduled
+  if (p.counters != nullptr && blockIdx.x == 0)
+    for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
+      p.counters[i] = 0u;
+
+  if (warp == 0 && lane == 0) {
+    ptx::mbar_init(q_full, 1);
+    ptx::mbar_init(q_empty, 1);
+    for (int i = 0; i < kStages; ++i) {
+      ptx::mbar_init(k_full + i, 1);
+      ptx::mbar_init(k_empty + i, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      ptx::mbar_init(a_full + i, 1);
+      ptx::mbar_init(a_empty + i, kEpiWarps);
+    }
+    ptx::fence_barrier_init();
+    ptx::fence_proxy_async_smem();
+    ptx::prefetch_tensormap(&tmQ);
+    ptx::prefetch_tensormap(&tmK);
+  }
+  if (warp == 1) ptx::tmem_alloc(tmem_slot, 256);
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  uint64_t limit = kWaitNs;
+
+  if (warp == 0) {
+    // ================= TMA producer: per unit the 128 text rows, then every
+    // key tile of sweep 1 and of sweep 2 through the ring
+    if (lane == 0) {
+      int ld = 0, u = 0;
+      for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x, ++u) {
+        const SGeo g = stream_geo(p, unit);
+        if (!g.ok) E2S_DEV_FLAG(p.status, E2S_ERR_SHAPE);
+        if (u > 0 && !ptx::mbar_wait(q_empty, (u - 1) & 1, limit, p.status))
+          limit = kWaitNsAfterFault;
+        if (g.n1 + g.n2 > 0) {
+          const int qrow = g.l * la.sum_text + g.x0;
+          ptx::mbar_arrive_expect_tx(q_full, (uint32_t)kTileBytes);
+          ptx::tma_load_3d(q_sm, &tmQ, q_full, 0, g.h, qrow);
+          ptx::tma_load_3d(q_sm + kHalfBytes, &tmQ, q_full, 64, g.h, qrow);
+        } else {
+          ptx::mbar_arrive(q_full);
+        }
+        for (int j = 0; j < g.n1 + g.n2; ++j, ++ld) {
+          const int s = ld % kStages;
+          if (ld >= kStages && !ptx::mbar_wait(k_empty + s, (ld / kStages - 1) & 1, limit, p.status))
+            limit = kWaitNsAfterFault;
+          const int key0 = j < g.n1 ? kTileKeys * j : g.S + kTileKeys * (j - g.n1);
+          const int krow = g.l * la.sum_T + g.t0 + key0;
+          ptx::mbar_arrive_expect_tx(k_full + s, (uint32_t)kTileBytes);
+          ptx::tma_load_3d(k_sm + s * kTileBytes, &tmK, k_full + s, 0, g.kvh, krow);
+          ptx::tma_load_3d(k_sm + s * kTileBytes + kHalfBytes, &tmK, k_full + s, 64, g.kvh, krow);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ================= MMA issuer: D[t][key] into accumulator buffer tc % 2
+    if (lane == 0) {
+      const uint32_t idesc = ptx::idesc_bf16_f32(kRows, kTileKeys);
+      const uint32_t a_base = ptx::smem_addr(q_sm);
+      int ld = 0, tc = 0, u = 0;
+      for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x, ++u) {
+        const SGeo g = stream_geo(p, unit);
+        if (!ptx::mbar_wait(q_full, u & 1, limit, p.status)) limit = kWaitNsAfterFault;
+        for (int j = 0; j < g.n1 + g.n2; ++j, ++ld, ++tc) {
+          const int s = ld % kStages, buf = tc & 1;
+          if (!ptx::mbar_wait(k_full + s, (ld / kStages) & 1, limit, p.status))
+            limit = kWaitNsAfterFault;
+          if (tc >= 2 && !ptx::mbar_wait(a_empty + buf, (tc / 2 - 1) & 1, limit, p.status))
+            limit = kWaitNsAfterFault;
+          ptx::tc_fence_after();
+          const uint32_t b_base = ptx::smem_addr(k_sm + s * kTileBytes);
+          const uint32_t d = tmem + (uint32_t)(buf * kTileKeys);
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks) {
+            const uint32_t half = ks >> 2, kk = ks & 3;
+            const uint64_t ad = ptx::sdesc_sw128(a_base + half * kHalfBytes + kk * 32u);
+            const uint64_t bd = ptx::sdesc_sw128(b_base + half * kHalfBytes + kk * 32u);
+            ptx::mma_bf16(d, ad, bd, idesc, ks > 0 ? 1u : 0u);
+          }
+          ptx::mma_commit(k_empty + s);   // the producer may refill the stage
+          ptx::mma_commit(a_full + buf);  // the epilogue may read the buffer
+        }
+        ptx::mma_commit(q_empty);   // every MMA of the unit is done with Q
+      }
+    }
+  } else {
+    // ================= epilogue (16 warps)
+    const int ew = warp - 2;
+    const int q4 = warp & 3;                 // TMEM lane quarter: text rows 32*q4 ..
+    const int cg = ew >> 2;                  // column group: keys 32*cg .. of each tile
+    const int t = q4 * 32 + lane;            // this lane's text row
+    const uint32_t lane_base = (uint32_t)(q4 * 32) << 16;
+    const int et = threadIdx.x - 64;
+    int tc = 0;
+    for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x) {
+      const SGeo g = stream_geo(p, unit);
+      const bool rows_live = q4 * 32 < g.NT;      // warp-uniform
+      const bool tvalid = t < g.NT;
+      const int lim = tvalid ? g.S + g.NV + t : -1;   // last key this row sees
+      const float inv_nt = 1.f / (float)max(g.NT, 1);
+      const int NV = g.ok ? g.NV : 0;
+      // ---- sweep 1: running (max, sum) per row over this warp's columns
+      float m = kNegBig, ssum = 0.f;
+      for (int j = 0; j < g.n1; ++j, ++tc) {
+        const int buf = tc & 1;
+        if (!ptx::mbar_wait(a_full + buf, (tc / 2) & 1, limit, p.status)) limit = kWaitNsAfterFault;
+        ptx::tc_fence_after();
+        if (rows_live) {
+#pragma unroll
+          for (int ch = 0; ch < 2; ++ch) {
+            const int c16 = cg * 32 + ch * 16;
+            const int key0 = kTileKeys * j + c16;
+            float x[16];
+            ptx::tmem_ld16(tmem + lane_base + (uint32_t)(buf * kTileKeys + c16), x);
+            if (key0 <= lim) {   // the row sees at least the chunk's first key
+              float cmax = kNegBig;
+              if (key0 + 15 <= lim) {
+#pragma unroll
+                for (int jj = 0; jj < 16; ++jj) cmax = fmaxf(cmax, x[jj]);
+              } else {
+#pragma unroll
+                for (int jj = 0; jj < 16; ++jj)
+                  if (key0 + jj <= lim) cmax = fmaxf(cmax, x[jj]);
+              }
+              const float mnew = fmaxf(m, cmax * p.scale_log2);
+              float acc = ssum * fast_ex2(m - mnew);
+#pragma unroll
+              for (int jj = 0; jj < 16; ++jj)
+                if (key0 + jj <= lim) acc += fast_ex2(fmaf(x[jj], p.scale_log2, -mnew));
+              ssum = acc;
+              m = mnew;
+            }
+          }
+        }
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(a_empty + buf);
+      }
+      // ---- merge the four column groups: lse per row (log2 domain)
+      float lse = 0.f;
+      if (causal) {
+        ms[cg * kRows + t] = make_float2(m, ssum);
+        ptx::named_bar(1, kEpiThreads);
+        float M = kNegBig;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) M = fmaxf(M, ms[c * kRows + t].x);
+        float L = 0.f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const float2 v = ms[c * kRows + t];
+          L += v.y * fast_ex2(v.x - M);
+        }
+        lse = L > 0.f ? M + __log2f(L) : kNegBig;
+      }
+      // ---- sweep 2: scores of the visual keys
+      for (int j = 0; j < g.n2; ++j, ++tc) {
+        const int buf = tc & 1;
+        float* cp = cps + (j & 1) * 4 * kTileKeys;
+        if (!ptx::mbar_wait(a_full + buf, (tc / 2) & 1, limit, p.status)) limit = kWaitNsAfterFault;
+        ptx::tc_fence_after();
+#pragma unroll
+        for (int ch = 0; ch < 2; ++ch) {
+          const int c16 = cg * 32 + ch * 16;
+          const int n0 = kTileKeys * j + c16;   // visual index of the chunk's first key
+          float r = 0.f;
+          if (rows_live) {
+            float x[16];
+            ptx::tmem_ld16(tmem + lane_base + (uint32_t)(buf * kTileKeys + c16), x);
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj) {
+              const bool valid = tvalid && n0 + jj < NV;
+              x[jj] = valid ? (causal ? fast_ex2(fmaf(x[jj], p.scale_log2, -lse)) : x[jj] * p.scale)
+                            : 0.f;
+            }
+            r = reduce_scatter16(x, lane, AddOp());
+          }
+          if ((lane & 1) == 0) cp[q4 * kTileKeys + c16 + (lane >> 1)] = r;
+        }
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(a_empty + buf);
+        ptx::named_bar(2 + cg, 128);   // the four lane quarters of this column group
+        if (q4 == 0) {
+          const int col = cg * 32 + lane;
+          const int n = kTileKeys * j + col;
+          if (n < NV) {
+            const float a = (((cp[col] + cp[kTileKeys + col]) + cp[2 * kTileKeys + col]) +
+                             cp[3 * kTileKeys + col]) * inv_nt;
+            as[n] = a;
+            p.a_out[((size_t)g.l * la.H + g.h) * (size_t)la.sum_vis + g.v0 + n] = a;
+          }
+        }
+      }
+      // ---- statistics of the unit's visual scores for Eq. 8
+      ptx::named_bar(1, kEpiThreads);   // every as[] written
+      float ls = 0.f, lm = kNegBig;
+      for (int n = et; n < NV; n += kEpiThreads) {
+        ls += as[n];
+        lm = fmaxf(lm, as[n] * kLog2e);
+      }
+      ls = warp_reduce(ls, [](float x, float y) { return x + y; });
+      lm = warp_reduce(lm, [](float x, float y) { return fmaxf(x, y); });
+      if (lane == 0) red[ew] = make_float2(ls, lm);
+      ptx::named_bar(1, kEpiThreads);
+      float S = 0.f, M = kNegBig;
+      for (int w = 0; w < kEpiWarps; ++w) {
+        S += red[w].x;
+        M = fmaxf(M, red[w].y);
+      }
+      float le = 0.f;
+      for (int n = et; n < NV; n += kEpiThreads) le += fast_ex2(fmaf(as[n], kLog2e, -M));
+      le = warp_reduce(le, [](float x, float y) { return x + y; });
+      if (lane == 0) red[kEpiWarps + ew] = make_float2(le, 0.f);
+      ptx::named_bar(1, kEpiThreads);
+      if (et == 0 && g.ok) {
+        float E = 0.f;
+        for (int w = 0; w < kEpiWarps; ++w) E += red[kEpiWarps + w].x;
+        p.stats[((size_t)g.b * la.L + g.l) * la.H + g.h] = stats_entry(S, M, E);
+      }
+      // ms, cps, as and red are rewritten by the next unit only after this barrier
+      ptx::named_bar(1, kEpiThreads);
+    }
+  }
+
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, 256);
+  }
+}
+
+}  // namespace
+
+// Whether the streaming kernel can take this launch: at most 128 text rows per
+// image and the unit's scores in shared memory.
+bool score_stream_fits(const LayoutArgs& la) {
+  if (la.max_text > kRows || la.H % la.H_kv) return false;
+  int dev = 0, optin = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  return (int)(stream_plan(la.max_vis).total + 1024) <= optin;
+}
+
+cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
+                                const void* k, int64_t k_stride, float* a_out, float4* stats,
+                                uint32_t* counters, uint32_t* status, cudaStream_t st) {
+  StreamArgs p;
+  p.la = la;
+  p.mode = mode;
+  p.group = la.H / la.H_kv;
+  p.num_units = la.B * la.L * la.H;
+  p.scale = 1.0f / sqrtf(128.0f);
+  p.scale_log2 = 1.4426950408889634f / sqrtf(128.0f);
+  p.a_out = a_out;
+  p.stats = stats;
+  p.counters = counters;
+  p.status = status;
+  if (p.num_units == 0 || la.sum_vis == 0) return cudaSuccess;
+  CUtensorMap tmQ, tmK;
+  if (!make_score_map(&tmQ, q, la.H, (int64_t)la.L * la.sum_text, q_stride, kRows) ||
+      !make_score_map(&tmK, k, la.H_kv, (int64_t)la.L * la.sum_T, k_stride, kTileKeys))
+    return cudaErrorInvalidValue;
+  const size_t smem = stream_plan(la.max_vis).total + 1024;
+  return launch_kernel(score_stream_kernel, dim3((unsigned)std::min(p.num_units, sm_count())),
+                       dim3(kThreads), smem, st, 0, false, tmQ, tmK, p);
+}
+
+}  // namespace e2s

@@ -507,6 +507,9 @@ cudaError_t launch_score_tc(const LayoutArgs& la, int mode, const void* q, int64
   if (score_unit_fits(la, mode))
     return launch_score_unit(la, mode, q, q_stride, k, k_stride, a_out, stats, counters, status,
                              st);
+  if (score_stream_fits(la))
+    return launch_score_stream(la, mode, q, q_stride, k, k_stride, a_out, stats, counters, status,
+                               st);
   TcArgs p;
   p.la = la;
   p.group = la.H / la.H_kv;
