@@ -74,8 +74,9 @@ bool score_stream_fits(const LayoutArgs& la);
 cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                                 const void* k, int64_t k_stride, float* a_out, float4* stats,
                                 uint32_t* counters, uint32_t* status, cudaStream_t st);
-// Persistent single-CTA-per-unit score kernel and its applicability test.
+// Persistent single-CTA-per-unit score kernel and its applicability tests.
 bool score_unit_fits(const LayoutArgs& la, int mode);
+bool score_unit_single_group(const LayoutArgs& la, int mode);
 cudaError_t launch_score_unit(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                               const void* k, int64_t k_stride, float* a_out, float4* stats,
                               uint32_t* counters, uint32_t* status, cudaStream_t st);

@@ -504,12 +504,21 @@ cudaError_t launch_score_tc(const LayoutArgs& la, int mode, const void* q, int64
                             uint32_t* counters, uint32_t* status, cudaStream_t st,
                             int* unsupported) {
   *unsupported = 0;
-  if (score_unit_fits(la, mode))
+  // kernel choice (measured): the persistent single-CTA kernel when every
+  // unit's logits fit TMEM in one column group (short sequences, e.g. one
+  // LLaVA image); the streaming kernel for longer sequences, GQA and batched
+  // ragged text (up to 128 text rows); the column-group kernel above 128 text
+  // rows while the K tiles fit shared memory; the cluster kernel otherwise
+  const bool unit = score_unit_fits(la, mode);
+  if (unit && score_unit_single_group(la, mode))
     return launch_score_unit(la, mode, q, q_stride, k, k_stride, a_out, stats, counters, status,
                              st);
   if (score_stream_fits(la))
     return launch_score_stream(la, mode, q, q_stride, k, k_stride, a_out, stats, counters, status,
                                st);
+  if (unit)
+    return launch_score_unit(la, mode, q, q_stride, k, k_stride, a_out, stats, counters, status,
+                             st);
   TcArgs p;
   p.la = la;
   p.group = la.H / la.H_kv;

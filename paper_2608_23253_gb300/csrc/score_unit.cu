@@ -821,6 +821,11 @@ static int unit_ntg(const LayoutArgs& la, int mode) {
   return std::min(ntp_max, (512 / tiles) / 16 * 16);
 }
 
+// Whether every unit is a single column group (score_unit_kernel).
+bool score_unit_single_group(const LayoutArgs& la, int mode) {
+  return unit_ntg(la, mode) >= ((std::max(la.max_text, 1) + 15) / 16) * 16;
+}
+
 // Whether the persistent kernel can take this launch (see the file comment).
 bool score_unit_fits(const LayoutArgs& la, int mode) {
   if (la.H != la.H_kv) return false;

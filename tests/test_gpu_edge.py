@@ -66,6 +66,16 @@ def test_max_text_rows(mode):
 
 
 @pytest.mark.parametrize("mode", ["causal", "eq1"])
+def test_text_rows_in_column_groups(mode):
+    """Short sequences with more than 128 text rows: the persistent kernel runs
+    each unit's text rows in two column groups that share the resident K tiles."""
+    ims = [ImageSpec(35, 16, 16, 200, 20, 3, 28), ImageSpec(35, 12, 12, 150, 10, 2, 16),
+           ImageSpec(3, 8, 8, 40, 5, 0, 7)]
+    inp = synth.make_inputs(_spec(ims, L=2, H=4, H_kv=4, cfg_id=95), with_payload=False)
+    _check(inp, run_gpu(inp, mode), run_oracle(inp, mode))
+
+
+@pytest.mark.parametrize("mode", ["causal", "eq1"])
 def test_gqa_split_head_groups(mode):
     """Group of 7 query heads with 128 text rows: the heads of a kv head are split over CTAs."""
     ims = [ImageSpec(35, 16, 16, 128, 20, 3, 28), ImageSpec(35, 24, 32, 100, 50, 3, 85)]
