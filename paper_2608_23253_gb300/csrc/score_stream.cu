@@ -17,7 +17,8 @@
 //           reduce-scatter inside a warp, then the four lane quarters in a
 //           fixed order through shared memory), a[key] = sum_t P / N_T.
 // EQ1 mode has no sweep 1 and sums s / sqrt(d) / N_T in sweep 2.
-// K tiles stream through a 4-stage ring (TMA producer warp), the accumulator
+// K tiles stream through a ring of as many stages as shared memory holds
+// (TMA producer warp; deep enough to cover the load latency), the accumulator
 // is double-buffered in TMEM (MMA warp), so loads, MMAs and the epilogue of
 // consecutive tiles overlap.
 //
@@ -42,7 +43,7 @@ constexpr int kRows = 128;                    // text rows per unit (M)
 constexpr int kTileKeys = 128;                // keys per tile (N)
 constexpr int kHalfBytes = 128 * 128;         // 128 rows x 64 bf16
 constexpr int kTileBytes = 2 * kHalfBytes;    // one 128 x 128 bf16 operand
-constexpr int kStages = 4;
+constexpr int kMaxStages = 8;                 // K ring depth: as many as shared memory holds
 constexpr int kEpiWarps = 16;
 constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr int kThreads = 64 + kEpiThreads;
@@ -53,6 +54,7 @@ constexpr float kLog2e = 1.4426950408889634f;
 struct StreamArgs {
   LayoutArgs la;
   int mode;
+  int stages;           // K ring stages (2 .. kMaxStages)
   int group;            // query heads per kv head
   int num_units;
   float scale;          // 1 / sqrt(d)
@@ -64,20 +66,19 @@ struct StreamArgs {
 };
 
 struct SPlan {
-  uint32_t q, k, bars, slot, ms, cps, red, as, total;
+  uint32_t q, k, bars, slot, ms, cps, red, total;
 };
 
-__host__ __device__ inline SPlan stream_plan(int max_vis) {
+__host__ __device__ inline SPlan stream_plan(int stages) {
   SPlan s;
   s.q = 0;                                              // [2 halves][128 rows][128 B]
-  s.k = (uint32_t)kTileBytes;                           // [kStages][tile]
-  s.bars = s.k + (uint32_t)kStages * kTileBytes;        // 2 + 2*kStages + 4 mbarriers
-  s.slot = s.bars + 8u * (uint32_t)(2 + 2 * kStages + 4);
+  s.k = (uint32_t)kTileBytes;                           // [stages][tile]
+  s.bars = s.k + (uint32_t)stages * kTileBytes;         // 2 + 2*kMaxStages + 4 mbarriers
+  s.slot = s.bars + 8u * (uint32_t)(2 + 2 * kMaxStages + 4);
   s.ms = (s.slot + 16u + 15u) & ~15u;                   // [4][128] float2 (max, sum)
   s.cps = s.ms + 4u * kRows * 8u;                       // [2][4][128] column partials
-  s.red = s.cps + 2u * 4u * kTileKeys * 4u;             // [2][kEpiWarps] float2
-  s.as = s.red + 2u * kEpiWarps * 8u;                   // [max_vis] the unit's scores
-  s.total = s.as + (uint32_t)(max_vis > 1 ? max_vis : 1) * 4u;
+  s.red = s.cps + 2u * 4u * kTileKeys * 4u;             // [4] float4 statistics partials
+  s.total = s.red + 4u * 16u;
   return s;
 }
 
@@ -142,20 +143,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const LayoutArgs& la = p.la;
-  const SPlan plan = stream_plan(la.max_vis);
+  const SPlan plan = stream_plan(p.stages);
   uint8_t* q_sm = smem + plan.q;
   uint8_t* k_sm = smem + plan.k;
   uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + plan.bars);
   uint64_t* q_empty = q_full + 1;
-  uint64_t* k_full = q_empty + 1;          // [kStages]
-  uint64_t* k_empty = k_full + kStages;    // [kStages]
-  uint64_t* a_full = k_empty + kStages;    // [2] accumulator buffer ready
+  uint64_t* k_full = q_empty + 1;          // [kMaxStages]
+  uint64_t* k_empty = k_full + kMaxStages; // [kMaxStages]
+  uint64_t* a_full = k_empty + kMaxStages; // [2] accumulator buffer ready
   uint64_t* a_empty = a_full + 2;          // [2] accumulator buffer read
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + plan.slot);
   float2* ms = reinterpret_cast<float2*>(smem + plan.ms);
   float* cps = reinterpret_cast<float*>(smem + plan.cps);
-  float2* red = reinterpret_cast<float2*>(smem + plan.red);
-  float* as = reinterpret_cast<float*>(smem + plan.as);
+  float4* red = reinterpret_cast<float4*>(smem + plan.red);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
@@ -167,7 +167,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0 && lane == 0) {
     ptx::mbar_init(q_full, 1);
     ptx::mbar_init(q_empty, 1);
-    for (int i = 0; i < kStages; ++i) {
+    for (int i = 0; i < kMaxStages; ++i) {
       ptx::mbar_init(k_full + i, 1);
       ptx::mbar_init(k_empty + i, 1);
     }
@@ -206,8 +206,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           ptx::mbar_arrive(q_full);
         }
         for (int j = 0; j < g.n1 + g.n2; ++j, ++ld) {
-          const int s = ld % kStages;
-          if (ld >= kStages && !ptx::mbar_wait(k_empty + s, (ld / kStages - 1) & 1, limit, p.status))
+          const int s = ld % p.stages;
+          if (ld >= p.stages &&
+              !ptx::mbar_wait(k_empty + s, (ld / p.stages - 1) & 1, limit, p.status))
             limit = kWaitNsAfterFault;
           const int key0 = j < g.n1 ? kTileKeys * j : g.S + kTileKeys * (j - g.n1);
           const int krow = g.l * la.sum_T + g.t0 + key0;
@@ -227,8 +228,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const SGeo g = stream_geo(p, unit);
         if (!ptx::mbar_wait(q_full, u & 1, limit, p.status)) limit = kWaitNsAfterFault;
         for (int j = 0; j < g.n1 + g.n2; ++j, ++ld, ++tc) {
-          const int s = ld % kStages, buf = tc & 1;
-          if (!ptx::mbar_wait(k_full + s, (ld / kStages) & 1, limit, p.status))
+          const int s = ld % p.stages, buf = tc & 1;
+          if (!ptx::mbar_wait(k_full + s, (ld / p.stages) & 1, limit, p.status))
             limit = kWaitNsAfterFault;
           if (tc >= 2 && !ptx::mbar_wait(a_empty + buf, (tc / 2 - 1) & 1, limit, p.status))
             limit = kWaitNsAfterFault;
@@ -277,16 +278,24 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int key0 = kTileKeys * j + c16;
             float x[16];
             ptx::tmem_ld16(tmem + lane_base + (uint32_t)(buf * kTileKeys + c16), x);
-            if (key0 <= lim) {   // the row sees at least the chunk's first key
-              float cmax = kNegBig;
-              if (key0 + 15 <= lim) {
+            if (key0 + 15 <= lim) {   // the row sees the whole chunk
+              float cmax = x[0];
 #pragma unroll
-                for (int jj = 0; jj < 16; ++jj) cmax = fmaxf(cmax, x[jj]);
-              } else {
+              for (int jj = 1; jj < 16; ++jj) cmax = fmaxf(cmax, x[jj]);
+              const float mnew = fmaxf(m, cmax * p.scale_log2);
+              float acc0 = ssum * fast_ex2(m - mnew), acc1 = 0.f;
 #pragma unroll
-                for (int jj = 0; jj < 16; ++jj)
-                  if (key0 + jj <= lim) cmax = fmaxf(cmax, x[jj]);
+              for (int jj = 0; jj < 16; jj += 2) {
+                acc0 += fast_ex2(fmaf(x[jj], p.scale_log2, -mnew));
+                acc1 += fast_ex2(fmaf(x[jj + 1], p.scale_log2, -mnew));
               }
+              ssum = acc0 + acc1;
+              m = mnew;
+            } else if (key0 <= lim) {   // the chunk straddles the row's last key
+              float cmax = kNegBig;
+#pragma unroll
+              for (int jj = 0; jj < 16; ++jj)
+                if (key0 + jj <= lim) cmax = fmaxf(cmax, x[jj]);
               const float mnew = fmaxf(m, cmax * p.scale_log2);
               float acc = ssum * fast_ex2(m - mnew);
 #pragma unroll
@@ -317,7 +326,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         lse = L > 0.f ? M + __log2f(L) : kNegBig;
       }
-      // ---- sweep 2: scores of the visual keys
+      // ---- sweep 2: scores of the visual keys; the q4 == 0 warps also keep
+      // the statistics of Eq. 8 online (sum, max of a*log2e, sum of exp2)
+      float st_s = 0.f, st_m = kNegBig, st_e = 0.f;
       for (int j = 0; j < g.n2; ++j, ++tc) {
         const int buf = tc & 1;
         float* cp = cps + (j & 1) * 4 * kTileKeys;
@@ -331,11 +342,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (rows_live) {
             float x[16];
             ptx::tmem_ld16(tmem + lane_base + (uint32_t)(buf * kTileKeys + c16), x);
+            const bool full = tvalid && n0 + 15 < NV;
+            if (causal) {
+              if (full) {
 #pragma unroll
-            for (int jj = 0; jj < 16; ++jj) {
-              const bool valid = tvalid && n0 + jj < NV;
-              x[jj] = valid ? (causal ? fast_ex2(fmaf(x[jj], p.scale_log2, -lse)) : x[jj] * p.scale)
-                            : 0.f;
+                for (int jj = 0; jj < 16; ++jj) x[jj] = fast_ex2(fmaf(x[jj], p.scale_log2, -lse));
+              } else {
+#pragma unroll
+                for (int jj = 0; jj < 16; ++jj)
+                  x[jj] = (tvalid && n0 + jj < NV) ? fast_ex2(fmaf(x[jj], p.scale_log2, -lse)) : 0.f;
+              }
+            } else {
+#pragma unroll
+              for (int jj = 0; jj < 16; ++jj)
+                x[jj] = (tvalid && n0 + jj < NV) ? x[jj] * p.scale : 0.f;
             }
             r = reduce_scatter16(x, lane, AddOp());
           }
@@ -351,38 +371,37 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (n < NV) {
             const float a = (((cp[col] + cp[kTileKeys + col]) + cp[2 * kTileKeys + col]) +
                              cp[3 * kTileKeys + col]) * inv_nt;
-            as[n] = a;
             p.a_out[((size_t)g.l * la.H + g.h) * (size_t)la.sum_vis + g.v0 + n] = a;
+            const float al = a * kLog2e, mnew = fmaxf(st_m, al);
+            st_e = st_e * fast_ex2(st_m - mnew) + fast_ex2(al - mnew);
+            st_m = mnew;
+            st_s += a;
           }
         }
       }
-      // ---- statistics of the unit's visual scores for Eq. 8
-      ptx::named_bar(1, kEpiThreads);   // every as[] written
-      float ls = 0.f, lm = kNegBig;
-      for (int n = et; n < NV; n += kEpiThreads) {
-        ls += as[n];
-        lm = fmaxf(lm, as[n] * kLog2e);
+      // ---- statistics of the unit's visual scores: merge the 128 producing
+      // lanes (four warps) in a fixed order
+      if (q4 == 0) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          const float s2 = __shfl_xor_sync(0xffffffffu, st_s, o);
+          const float m2 = __shfl_xor_sync(0xffffffffu, st_m, o);
+          const float e2 = __shfl_xor_sync(0xffffffffu, st_e, o);
+          st_s += s2;
+          lse_merge(st_m, st_e, m2, e2);
+        }
+        if (lane == 0) red[cg] = make_float4(st_s, st_m, st_e, 0.f);
       }
-      ls = warp_reduce(ls, [](float x, float y) { return x + y; });
-      lm = warp_reduce(lm, [](float x, float y) { return fmaxf(x, y); });
-      if (lane == 0) red[ew] = make_float2(ls, lm);
-      ptx::named_bar(1, kEpiThreads);
-      float S = 0.f, M = kNegBig;
-      for (int w = 0; w < kEpiWarps; ++w) {
-        S += red[w].x;
-        M = fmaxf(M, red[w].y);
-      }
-      float le = 0.f;
-      for (int n = et; n < NV; n += kEpiThreads) le += fast_ex2(fmaf(as[n], kLog2e, -M));
-      le = warp_reduce(le, [](float x, float y) { return x + y; });
-      if (lane == 0) red[kEpiWarps + ew] = make_float2(le, 0.f);
       ptx::named_bar(1, kEpiThreads);
       if (et == 0 && g.ok) {
-        float E = 0.f;
-        for (int w = 0; w < kEpiWarps; ++w) E += red[kEpiWarps + w].x;
+        float S = 0.f, M = kNegBig, E = 0.f;
+        for (int c = 0; c < 4; ++c) {
+          S += red[c].x;
+          lse_merge(M, E, red[c].y, red[c].z);
+        }
         p.stats[((size_t)g.b * la.L + g.l) * la.H + g.h] = stats_entry(S, M, E);
       }
-      // ms, cps, as and red are rewritten by the next unit only after this barrier
+      // ms, cps and red are rewritten by the next unit only after this barrier
       ptx::named_bar(1, kEpiThreads);
     }
   }
@@ -397,14 +416,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-// Whether the streaming kernel can take this launch: at most 128 text rows per
-// image and the unit's scores in shared memory.
-bool score_stream_fits(const LayoutArgs& la) {
-  if (la.max_text > kRows || la.H % la.H_kv) return false;
+// K ring stages that fit the device's shared memory (0 if fewer than two).
+static int stream_stages() {
   int dev = 0, optin = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
   cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-  return (int)(stream_plan(la.max_vis).total + 1024) <= optin;
+  for (int st = kMaxStages; st >= 2; --st)
+    if ((int)(stream_plan(st).total + 1024) <= optin) return st;
+  return 0;
+}
+
+// Whether the streaming kernel can take this launch: at most 128 text rows.
+bool score_stream_fits(const LayoutArgs& la) {
+  return la.max_text <= kRows && la.H % la.H_kv == 0 && stream_stages() >= 2;
 }
 
 cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
@@ -413,6 +437,7 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
   StreamArgs p;
   p.la = la;
   p.mode = mode;
+  p.stages = stream_stages();
   p.group = la.H / la.H_kv;
   p.num_units = la.B * la.L * la.H;
   p.scale = 1.0f / sqrtf(128.0f);
@@ -426,7 +451,8 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
   if (!make_score_map(&tmQ, q, la.H, (int64_t)la.L * la.sum_text, q_stride, kRows) ||
       !make_score_map(&tmK, k, la.H_kv, (int64_t)la.L * la.sum_T, k_stride, kTileKeys))
     return cudaErrorInvalidValue;
-  const size_t smem = stream_plan(la.max_vis).total + 1024;
+  if (p.stages < 2) return cudaErrorInvalidValue;
+  const size_t smem = stream_plan(p.stages).total + 1024;
   return launch_kernel(score_stream_kernel, dim3((unsigned)std::min(p.num_units, sm_count())),
                        dim3(kThreads), smem, st, 0, false, tmQ, tmK, p);
 }
