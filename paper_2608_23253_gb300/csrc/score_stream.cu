@@ -3,8 +3,10 @@
 // causal-prefix probability reading).  Used when a unit's K does not fit in
 // shared memory or its heads share K (GQA), for at most 128 text rows.
 //
-// One CTA per SM loops over units (image, layer, query head); the query head
-// reads kv head h / (H / H_kv).  The MMA is transposed with respect to the
+// One CTA per SM loops over units (image, layer, query heads); query head h
+// reads kv head h / (H / H_kv).  When the text rows leave room, the query
+// heads of one kv head are stacked into the 128 TMEM lanes (two heads of up to
+// 64 rows, or four of up to 32), so that they share one stream of K tiles.  The MMA is transposed with respect to the
 // persistent single-CTA kernel: D[t][key] = Q[t][:] . K_tile[key][:] with the
 // 128 text rows on the TMEM lanes (M = 128) and 128 keys per tile on the
 // columns (N = 128), so each text row's softmax over its keys is lane-local:
@@ -56,6 +58,7 @@ struct StreamArgs {
   int mode;
   int stages;           // K ring stages (2 .. kMaxStages)
   int group;            // query heads per kv head
+  int upk;              // units per kv head: ceil(group / stacked heads)
   int num_units;
   float scale;          // 1 / sqrt(d)
   float scale_log2;     // log2(e) / sqrt(d)
@@ -77,8 +80,8 @@ __host__ __device__ inline SPlan stream_plan(int stages) {
   s.slot = s.bars + 8u * (uint32_t)(2 + 2 * kMaxStages + 4);
   s.ms = (s.slot + 16u + 15u) & ~15u;                   // [4][128] float2 (max, sum)
   s.cps = s.ms + 4u * kRows * 8u;                       // [2][4][128] column partials
-  s.red = s.cps + 2u * 4u * kTileKeys * 4u;             // [4] float4 statistics partials
-  s.total = s.red + 4u * 16u;
+  s.red = s.cps + 2u * 4u * kTileKeys * 4u;             // [4 heads][4] float4 statistics
+  s.total = s.red + 16u * 16u;
   return s;
 }
 
@@ -106,18 +109,29 @@ struct AddOp {
 
 // Geometry of one unit, derived identically by every warp role.
 struct SGeo {
-  int b, l, h, kvh, S, NV, NT, t0, x0, v0;
+  int b, l, h, kvh, nh, S, NV, NT, t0, x0, v0;   // heads h .. h + nh - 1
   int n1, n2;   // key tiles of sweep 1 (whole causal prefix) and sweep 2 (visual)
   bool ok;
 };
 
+template <int HPU>
 __device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit) {
   const LayoutArgs& la = p.la;
   SGeo g;
-  g.h = unit % la.H;
-  g.l = (unit / la.H) % la.L;
-  g.b = unit / (la.H * la.L);
-  g.kvh = g.h / p.group;
+  if (HPU == 1) {   // units are (image, layer, query head)
+    g.h = unit % la.H;
+    g.l = (unit / la.H) % la.L;
+    g.b = unit / (la.H * la.L);
+    g.kvh = g.h / p.group;
+    g.nh = 1;
+  } else {          // units are (image, layer, kv head, stack of query heads)
+    const int ug = unit % p.upk;
+    g.kvh = (unit / p.upk) % la.H_kv;
+    g.l = (unit / (p.upk * la.H_kv)) % la.L;
+    g.b = unit / (p.upk * la.H_kv * la.L);
+    g.h = g.kvh * p.group + ug * HPU;
+    g.nh = min(HPU, p.group - ug * HPU);
+  }
   g.S = __ldg(la.n_sys + g.b);
   g.NV = __ldg(la.n_vis + g.b);
   g.NT = __ldg(la.n_text + g.b);
@@ -125,7 +139,7 @@ __device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit) {
   g.x0 = __ldg(la.text_off + g.b);
   g.v0 = __ldg(la.vis_off + g.b);
   const int T = g.S + g.NV + g.NT;
-  g.ok = g.S >= 0 && g.NV >= 0 && g.NT >= 1 && g.NT <= kRows && T <= la.max_T &&
+  g.ok = g.S >= 0 && g.NV >= 0 && g.NT >= 1 && g.NT <= kRows / HPU && T <= la.max_T &&
          g.NV <= la.max_vis && __ldg(la.tok_off + g.b + 1) - g.t0 == T && g.t0 >= 0 &&
          g.t0 + T <= la.sum_T && __ldg(la.text_off + g.b + 1) - g.x0 == g.NT && g.x0 >= 0 &&
          g.x0 + g.NT <= la.sum_text && __ldg(la.vis_off + g.b + 1) - g.v0 == g.NV &&
@@ -136,6 +150,9 @@ __device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit) {
   return g;
 }
 
+// HPU: query heads stacked per unit (1, 2 or 4), fixed at compile time so that
+// the row mapping and the quarter sums are unrolled.
+template <int HPU>
 __global__ void __launch_bounds__(kThreads, 1)
     score_stream_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmK, const StreamArgs p) {
@@ -159,6 +176,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
+  constexpr int kRph = kRows / HPU;   // TMEM lanes per stacked head
+  constexpr int kQph = 4 / HPU;       // lane quarters per stacked head
   pdl_launch_dependents();   // every CTA is resident: the next kernel may be scheduled
   if (p.counters != nullptr && blockIdx.x == 0)
     for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
@@ -193,15 +212,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       int ld = 0, u = 0;
       for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x, ++u) {
-        const SGeo g = stream_geo(p, unit);
+        const SGeo g = stream_geo<HPU>(p, unit);
         if (!g.ok) E2S_DEV_FLAG(p.status, E2S_ERR_SHAPE);
         if (u > 0 && !ptx::mbar_wait(q_empty, (u - 1) & 1, limit, p.status))
           limit = kWaitNsAfterFault;
         if (g.n1 + g.n2 > 0) {
+          // kRows / HPU rows of each stacked head (an absent head repeats the last one;
+          // its rows are masked)
           const int qrow = g.l * la.sum_text + g.x0;
           ptx::mbar_arrive_expect_tx(q_full, (uint32_t)kTileBytes);
-          ptx::tma_load_3d(q_sm, &tmQ, q_full, 0, g.h, qrow);
-          ptx::tma_load_3d(q_sm + kHalfBytes, &tmQ, q_full, 64, g.h, qrow);
+#pragma unroll
+          for (int hs = 0; hs < HPU; ++hs) {
+            const int hq = g.h + min(hs, g.nh - 1);
+            const uint32_t off = (uint32_t)(hs * kRph) * 128u;
+            ptx::tma_load_3d(q_sm + off, &tmQ, q_full, 0, hq, qrow);
+            ptx::tma_load_3d(q_sm + kHalfBytes + off, &tmQ, q_full, 64, hq, qrow);
+          }
         } else {
           ptx::mbar_arrive(q_full);
         }
@@ -225,7 +251,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t a_base = ptx::smem_addr(q_sm);
       int ld = 0, tc = 0, u = 0;
       for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x, ++u) {
-        const SGeo g = stream_geo(p, unit);
+        const SGeo g = stream_geo<HPU>(p, unit);
         if (!ptx::mbar_wait(q_full, u & 1, limit, p.status)) limit = kWaitNsAfterFault;
         for (int j = 0; j < g.n1 + g.n2; ++j, ++ld, ++tc) {
           const int s = ld % p.stages, buf = tc & 1;
@@ -254,14 +280,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int ew = warp - 2;
     const int q4 = warp & 3;                 // TMEM lane quarter: text rows 32*q4 ..
     const int cg = ew >> 2;                  // column group: keys 32*cg .. of each tile
-    const int t = q4 * 32 + lane;            // this lane's text row
+    const int lrow = q4 * 32 + lane;         // this lane's TMEM row
     const uint32_t lane_base = (uint32_t)(q4 * 32) << 16;
     const int et = threadIdx.x - 64;
     int tc = 0;
     for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x) {
-      const SGeo g = stream_geo(p, unit);
-      const bool rows_live = q4 * 32 < g.NT;      // warp-uniform
-      const bool tvalid = t < g.NT;
+      const SGeo g = stream_geo<HPU>(p, unit);
+      // TMEM row lrow holds text row t of stacked head hs
+      const int hs = lrow / kRph, t = lrow - hs * kRph;
+      const bool rows_live = hs < g.nh && (q4 * 32) % kRph < g.NT;   // warp-uniform
+      const bool tvalid = hs < g.nh && t < g.NT;
       const int lim = tvalid ? g.S + g.NV + t : -1;   // last key this row sees
       const float inv_nt = 1.f / (float)max(g.NT, 1);
       const int NV = g.ok ? g.NV : 0;
@@ -313,21 +341,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---- merge the four column groups: lse per row (log2 domain)
       float lse = 0.f;
       if (causal) {
-        ms[cg * kRows + t] = make_float2(m, ssum);
+        ms[cg * kRows + lrow] = make_float2(m, ssum);
         ptx::named_bar(1, kEpiThreads);
         float M = kNegBig;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) M = fmaxf(M, ms[c * kRows + t].x);
+        for (int c = 0; c < 4; ++c) M = fmaxf(M, ms[c * kRows + lrow].x);
         float L = 0.f;
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
-          const float2 v = ms[c * kRows + t];
+          const float2 v = ms[c * kRows + lrow];
           L += v.y * fast_ex2(v.x - M);
         }
         lse = L > 0.f ? M + __log2f(L) : kNegBig;
       }
-      // ---- sweep 2: scores of the visual keys; the q4 == 0 warps also keep
-      // the statistics of Eq. 8 online (sum, max of a*log2e, sum of exp2)
+      // ---- sweep 2: scores of the visual keys; the first lane quarter of each
+      // stacked head also keeps that head's statistics of Eq. 8 online (sum,
+      // max of a*log2e, sum of exp2)
       float st_s = 0.f, st_m = kNegBig, st_e = 0.f;
       for (int j = 0; j < g.n2; ++j, ++tc) {
         const int buf = tc & 1;
@@ -365,13 +394,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(a_empty + buf);
         ptx::named_bar(2 + cg, 128);   // the four lane quarters of this column group
-        if (q4 == 0) {
+        if (q4 % kQph == 0 && hs < g.nh) {
           const int col = cg * 32 + lane;
           const int n = kTileKeys * j + col;
           if (n < NV) {
-            const float a = (((cp[col] + cp[kTileKeys + col]) + cp[2 * kTileKeys + col]) +
-                             cp[3 * kTileKeys + col]) * inv_nt;
-            p.a_out[((size_t)g.l * la.H + g.h) * (size_t)la.sum_vis + g.v0 + n] = a;
+            float a = cp[q4 * kTileKeys + col];
+#pragma unroll
+            for (int k = 1; k < kQph; ++k) a += cp[(q4 + k) * kTileKeys + col];
+            a *= inv_nt;
+            p.a_out[((size_t)g.l * la.H + g.h + hs) * (size_t)la.sum_vis + g.v0 + n] = a;
             const float al = a * kLog2e, mnew = fmaxf(st_m, al);
             st_e = st_e * fast_ex2(st_m - mnew) + fast_ex2(al - mnew);
             st_m = mnew;
@@ -379,9 +410,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      // ---- statistics of the unit's visual scores: merge the 128 producing
-      // lanes (four warps) in a fixed order
-      if (q4 == 0) {
+      // ---- statistics of each head's visual scores: merge the 128 producing
+      // lanes of the head (four warps, one per column group) in a fixed order
+      if (q4 % kQph == 0) {
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
           const float s2 = __shfl_xor_sync(0xffffffffu, st_s, o);
@@ -390,16 +421,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           st_s += s2;
           lse_merge(st_m, st_e, m2, e2);
         }
-        if (lane == 0) red[cg] = make_float4(st_s, st_m, st_e, 0.f);
+        if (lane == 0) red[hs * 4 + cg] = make_float4(st_s, st_m, st_e, 0.f);
       }
       ptx::named_bar(1, kEpiThreads);
-      if (et == 0 && g.ok) {
+      if (et < g.nh && g.ok) {   // thread et merges stacked head et
         float S = 0.f, M = kNegBig, E = 0.f;
         for (int c = 0; c < 4; ++c) {
-          S += red[c].x;
-          lse_merge(M, E, red[c].y, red[c].z);
+          const float4 r4 = red[et * 4 + c];
+          S += r4.x;
+          lse_merge(M, E, r4.y, r4.z);
         }
-        p.stats[((size_t)g.b * la.L + g.l) * la.H + g.h] = stats_entry(S, M, E);
+        p.stats[((size_t)g.b * la.L + g.l) * la.H + g.h + et] = stats_entry(S, M, E);
       }
       // ms, cps and red are rewritten by the next unit only after this barrier
       ptx::named_bar(1, kEpiThreads);
@@ -439,7 +471,12 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
   p.mode = mode;
   p.stages = stream_stages();
   p.group = la.H / la.H_kv;
-  p.num_units = la.B * la.L * la.H;
+  // stack the query heads of one kv head into the 128 TMEM lanes when their
+  // text rows leave room (64 rows: two heads, 32 rows: four)
+  int hpu = 1;
+  while (hpu < 4 && hpu * 2 <= p.group && la.max_text <= kRows / (hpu * 2)) hpu *= 2;
+  p.upk = (p.group + hpu - 1) / hpu;
+  p.num_units = la.B * la.L * la.H_kv * p.upk;
   p.scale = 1.0f / sqrtf(128.0f);
   p.scale_log2 = 1.4426950408889634f / sqrtf(128.0f);
   p.a_out = a_out;
@@ -448,13 +485,20 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
   p.status = status;
   if (p.num_units == 0 || la.sum_vis == 0) return cudaSuccess;
   CUtensorMap tmQ, tmK;
-  if (!make_score_map(&tmQ, q, la.H, (int64_t)la.L * la.sum_text, q_stride, kRows) ||
+  if (!make_score_map(&tmQ, q, la.H, (int64_t)la.L * la.sum_text, q_stride, kRows / hpu) ||
       !make_score_map(&tmK, k, la.H_kv, (int64_t)la.L * la.sum_T, k_stride, kTileKeys))
     return cudaErrorInvalidValue;
   if (p.stages < 2) return cudaErrorInvalidValue;
   const size_t smem = stream_plan(p.stages).total + 1024;
-  return launch_kernel(score_stream_kernel, dim3((unsigned)std::min(p.num_units, sm_count())),
-                       dim3(kThreads), smem, st, 0, false, tmQ, tmK, p);
+  const dim3 grid((unsigned)std::min(p.num_units, sm_count()));
+  if (hpu == 4)
+    return launch_kernel(score_stream_kernel<4>, grid, dim3(kThreads), smem, st, 0, false, tmQ,
+                         tmK, p);
+  if (hpu == 2)
+    return launch_kernel(score_stream_kernel<2>, grid, dim3(kThreads), smem, st, 0, false, tmQ,
+                         tmK, p);
+  return launch_kernel(score_stream_kernel<1>, grid, dim3(kThreads), smem, st, 0, false, tmQ, tmK,
+                       p);
 }
 
 }  // namespace e2s

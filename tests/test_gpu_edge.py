@@ -83,6 +83,20 @@ def test_gqa_split_head_groups(mode):
     _check(inp, run_gpu(inp, mode), run_oracle(inp, mode))
 
 
+@pytest.mark.parametrize("mode", ["causal", "eq1"])
+@pytest.mark.parametrize("H,H_kv,texts", [(14, 2, (64, 33, 1)), (16, 2, (32, 5, 17)),
+                                          (12, 4, (20, 32, 2)), (28, 4, (32, 9, 30))])
+def test_gqa_stacked_heads(mode, H, H_kv, texts):
+    """Short text with grouped-query heads: two (<= 64 rows) or four (<= 32 rows)
+    query heads of one kv head share the 128 accumulator rows, including groups
+    that do not divide evenly into stacks."""
+    grids = [(24, 32), (16, 16), (36, 36)]
+    ims = [ImageSpec(35, gh, gw, nt, max(1, gh * gw // 20), 2, max(1, gh * gw // 9))
+           for (gh, gw), nt in zip(grids, texts)]
+    inp = synth.make_inputs(_spec(ims, L=2, H=H, H_kv=H_kv, cfg_id=96), with_payload=False)
+    _check(inp, run_gpu(inp, mode), run_oracle(inp, mode))
+
+
 def test_all_equal_scores_tie_break():
     """Zero queries give equal logits everywhere: ties resolve to the lower index."""
     inp = config_inputs(0, None, None)
