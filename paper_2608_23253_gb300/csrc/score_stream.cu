@@ -6,18 +6,20 @@
 // One CTA per SM loops over units (image, layer, query heads); query head h
 // reads kv head h / (H / H_kv).  When the text rows leave room, the query
 // heads of one kv head are stacked into the 128 TMEM lanes (two heads of up to
-// 64 rows, or four of up to 32), so that they share one stream of K tiles.  The MMA is transposed with respect to the
-// persistent single-CTA kernel: D[t][key] = Q[t][:] . K_tile[key][:] with the
-// 128 text rows on the TMEM lanes (M = 128) and 128 keys per tile on the
-// columns (N = 128), so each text row's softmax over its keys is lane-local:
-//   sweep 1 every key tile of the causal prefix (keys 0 .. S+N_V+N_T-1):
+// 64 rows, or four of up to 32), so that they share one stream of K tiles.
+// Each key tile of 128 keys is one MMA with K = d = 128, in one of two
+// orientations:
+//   sweep 1 every key tile of the causal prefix (keys 0 .. S+N_V+N_T-1),
+//           D[t][key] = Q[t][:] . K[key][:], text rows on the TMEM lanes:
 //           each lane keeps a running (max, sum of exp2) of its row over the
 //           32 columns its warp reads -- no cross-lane work; at the end the
 //           four column groups merge into lse_t (log2 domain) per row;
 //   sweep 2 the visual tiles again (the MMAs are recomputed from re-streamed
-//           K): P = exp2(s - lse_t), column sums over the rows (butterfly
-//           reduce-scatter inside a warp, then the four lane quarters in a
-//           fixed order through shared memory), a[key] = sum_t P / N_T.
+//           K), D[key][t] = K[key][:] . Q[t][:], keys on the TMEM lanes and
+//           the text rows (rounded up to 16) on the columns: each lane sums
+//           P = exp2(s - lse_t) over the text rows of its column chunks, the
+//           chunk partials of a key are added in a fixed order through shared
+//           memory, and a[key] = sum_t P / N_T.
 // EQ1 mode has no sweep 1 and sums s / sqrt(d) / N_T in sweep 2.
 // K tiles stream through a ring of as many stages as shared memory holds
 // (TMA producer warp; deep enough to cover the load latency), the accumulator
@@ -25,8 +27,8 @@
 // consecutive tiles overlap.
 //
 // Warp roles (576 threads): warp 0 TMA producer, warp 1 TMEM allocator and MMA
-// issuer, warps 2-17 epilogue: warp w reads TMEM lane quarter w % 4 (text rows
-// 32*(w%4) ..) and column group (w - 2) / 4 (32 keys of each tile).
+// issuer, warps 2-17 epilogue: warp w reads TMEM lane quarter w % 4 and column
+// group (w - 2) / 4 (32 keys of each tile in sweep 1, column chunks in sweep 2).
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -69,7 +71,7 @@ struct StreamArgs {
 };
 
 struct SPlan {
-  uint32_t q, k, bars, slot, ms, cps, red, total;
+  uint32_t q, k, bars, slot, ms, lse, cps, red, total;
 };
 
 __host__ __device__ inline SPlan stream_plan(int stages) {
@@ -79,33 +81,12 @@ __host__ __device__ inline SPlan stream_plan(int stages) {
   s.bars = s.k + (uint32_t)stages * kTileBytes;         // 2 + 2*kMaxStages + 4 mbarriers
   s.slot = s.bars + 8u * (uint32_t)(2 + 2 * kMaxStages + 4);
   s.ms = (s.slot + 16u + 15u) & ~15u;                   // [4][128] float2 (max, sum)
-  s.cps = s.ms + 4u * kRows * 8u;                       // [2][4][128] column partials
-  s.red = s.cps + 2u * 4u * kTileKeys * 4u;             // [4 heads][4] float4 statistics
+  s.lse = s.ms + 4u * kRows * 8u;                       // [128] float lse per text row
+  s.cps = s.lse + kRows * 4u;                           // [2][8 chunks][128 keys] partials
+  s.red = s.cps + 2u * 8u * kTileKeys * 4u;             // [4 heads][4] float4 statistics
   s.total = s.red + 16u * 16u;
   return s;
 }
-
-template <int W, int MASK, class Op>
-__device__ __forceinline__ void rs_step(float (&x)[16], bool hi, Op op) {
-#pragma unroll
-  for (int i = 0; i < W; ++i) {
-    const float send = hi ? x[i] : x[i + W];
-    const float keep = hi ? x[i + W] : x[i];
-    x[i] = op(keep, __shfl_xor_sync(0xffffffffu, send, MASK));
-  }
-}
-// lane L ends with column L >> 1 of the 16, reduced over all 32 lanes
-template <class Op>
-__device__ __forceinline__ float reduce_scatter16(float (&x)[16], int lane, Op op) {
-  rs_step<8, 16>(x, lane & 16, op);
-  rs_step<4, 8>(x, lane & 8, op);
-  rs_step<2, 4>(x, lane & 4, op);
-  rs_step<1, 2>(x, lane & 2, op);
-  return op(x[0], __shfl_xor_sync(0xffffffffu, x[0], 1));
-}
-struct AddOp {
-  __device__ __forceinline__ float operator()(float a, float b) const { return a + b; }
-};
 
 // Geometry of one unit, derived identically by every warp role.
 struct SGeo {
@@ -150,6 +131,13 @@ __device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit) {
   return g;
 }
 
+// Text columns of the sweep-2 accumulator: the unit's rows rounded up to the
+// MMA's N granularity (16), or every lane of a stack of heads.
+template <int HPU>
+__device__ __forceinline__ int sweep2_cols(int NT) {
+  return HPU == 1 ? min(kRows, max(16, (NT + 15) & ~15)) : kRows;
+}
+
 // HPU: query heads stacked per unit (1, 2 or 4), fixed at compile time so that
 // the row mapping and the quarter sums are unrolled.
 template <int HPU>
@@ -171,13 +159,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* a_empty = a_full + 2;          // [2] accumulator buffer read
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + plan.slot);
   float2* ms = reinterpret_cast<float2*>(smem + plan.ms);
+  float* lse_s = reinterpret_cast<float*>(smem + plan.lse);
   float* cps = reinterpret_cast<float*>(smem + plan.cps);
   float4* red = reinterpret_cast<float4*>(smem + plan.red);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
   constexpr int kRph = kRows / HPU;   // TMEM lanes per stacked head
-  constexpr int kQph = 4 / HPU;       // lane quarters per stacked head
   pdl_launch_dependents();   // every CTA is resident: the next kernel may be scheduled
   if (p.counters != nullptr && blockIdx.x == 0)
     for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
@@ -245,13 +233,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else if (warp == 1) {
-    // ================= MMA issuer: D[t][key] into accumulator buffer tc % 2
+    // ================= MMA issuer into accumulator buffer tc % 2: sweep 1
+    // D[t][key] (text rows on the lanes), sweep 2 D[key][t] (keys on the lanes)
     if (lane == 0) {
-      const uint32_t idesc = ptx::idesc_bf16_f32(kRows, kTileKeys);
-      const uint32_t a_base = ptx::smem_addr(q_sm);
+      const uint32_t idesc1 = ptx::idesc_bf16_f32(kRows, kTileKeys);
+      const uint32_t q_base = ptx::smem_addr(q_sm);
       int ld = 0, tc = 0, u = 0;
       for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x, ++u) {
         const SGeo g = stream_geo<HPU>(p, unit);
+        const uint32_t idesc2 = ptx::idesc_bf16_f32(kTileKeys, sweep2_cols<HPU>(g.NT));
         if (!ptx::mbar_wait(q_full, u & 1, limit, p.status)) limit = kWaitNsAfterFault;
         for (int j = 0; j < g.n1 + g.n2; ++j, ++ld, ++tc) {
           const int s = ld % p.stages, buf = tc & 1;
@@ -260,7 +250,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (tc >= 2 && !ptx::mbar_wait(a_empty + buf, (tc / 2 - 1) & 1, limit, p.status))
             limit = kWaitNsAfterFault;
           ptx::tc_fence_after();
-          const uint32_t b_base = ptx::smem_addr(k_sm + s * kTileBytes);
+          const uint32_t k_base = ptx::smem_addr(k_sm + s * kTileBytes);
+          const bool sw2 = j >= g.n1;
+          const uint32_t a_base = sw2 ? k_base : q_base, b_base = sw2 ? q_base : k_base;
+          const uint32_t idesc = sw2 ? idesc2 : idesc1;
           const uint32_t d = tmem + (uint32_t)(buf * kTileKeys);
 #pragma unroll
           for (int ks = 0; ks < 8; ++ks) {
@@ -338,8 +331,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(a_empty + buf);
       }
-      // ---- merge the four column groups: lse per row (log2 domain)
-      float lse = 0.f;
+      // ---- merge the four column groups: lse per row (log2 domain), published
+      // per text row for sweep 2
       if (causal) {
         ms[cg * kRows + lrow] = make_float2(m, ssum);
         ptx::named_bar(1, kEpiThreads);
@@ -352,57 +345,77 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float2 v = ms[c * kRows + lrow];
           L += v.y * fast_ex2(v.x - M);
         }
-        lse = L > 0.f ? M + __log2f(L) : kNegBig;
+        if (cg == 0) lse_s[lrow] = L > 0.f ? M + __log2f(L) : kNegBig;
+        ptx::named_bar(1, kEpiThreads);
       }
-      // ---- sweep 2: scores of the visual keys; the first lane quarter of each
-      // stacked head also keeps that head's statistics of Eq. 8 online (sum,
-      // max of a*log2e, sum of exp2)
+      // ---- sweep 2: accumulator D[key][column], keys on the lanes, so each
+      // key's sum over text rows is lane-local.  Warp (q4, cg) reads column
+      // chunks cg and cg + 4 (16 columns each; chunk c holds text rows
+      // 16c % (128 / HPU) .. of stacked head 16c / (128 / HPU)) and leaves one
+      // partial per chunk and key; after the four warps of the lane quarter
+      // meet, warp cg sums the chunks of head cg in order and also keeps that
+      // head's statistics of Eq. 8 online (sum, max of a*log2e, sum of exp2).
+      const int nch = sweep2_cols<HPU>(g.NT) >> 4;
+      constexpr int kCph = kRph / 16;   // chunks per stacked head
+      const int head_chunks = min(kCph, (g.NT + 15) >> 4);
+      const float a_mul = causal ? inv_nt : p.scale * inv_nt;
       float st_s = 0.f, st_m = kNegBig, st_e = 0.f;
       for (int j = 0; j < g.n2; ++j, ++tc) {
         const int buf = tc & 1;
-        float* cp = cps + (j & 1) * 4 * kTileKeys;
+        float* cp = cps + (j & 1) * 8 * kTileKeys;
         if (!ptx::mbar_wait(a_full + buf, (tc / 2) & 1, limit, p.status)) limit = kWaitNsAfterFault;
         ptx::tc_fence_after();
 #pragma unroll
-        for (int ch = 0; ch < 2; ++ch) {
-          const int c16 = cg * 32 + ch * 16;
-          const int n0 = kTileKeys * j + c16;   // visual index of the chunk's first key
-          float r = 0.f;
-          if (rows_live) {
+        for (int r = 0; r < 2; ++r) {
+          const int c = cg + 4 * r;
+          const int ct = (c * 16) % kRph, chd = (c * 16) / kRph;   // first row, head
+          if (c < nch && chd < g.nh && ct < g.NT) {                 // warp-uniform
             float x[16];
-            ptx::tmem_ld16(tmem + lane_base + (uint32_t)(buf * kTileKeys + c16), x);
-            const bool full = tvalid && n0 + 15 < NV;
+            ptx::tmem_ld16(tmem + lane_base + (uint32_t)(buf * kTileKeys + c * 16), x);
+            float acc0 = 0.f, acc1 = 0.f;
             if (causal) {
-              if (full) {
+              const float4* l4 = reinterpret_cast<const float4*>(lse_s + c * 16);
+              float lv[16];
 #pragma unroll
-                for (int jj = 0; jj < 16; ++jj) x[jj] = fast_ex2(fmaf(x[jj], p.scale_log2, -lse));
+              for (int q = 0; q < 4; ++q) {
+                const float4 v = l4[q];
+                lv[4 * q] = v.x; lv[4 * q + 1] = v.y; lv[4 * q + 2] = v.z; lv[4 * q + 3] = v.w;
+              }
+              if (ct + 15 < g.NT) {
+#pragma unroll
+                for (int jj = 0; jj < 16; jj += 2) {
+                  acc0 += fast_ex2(fmaf(x[jj], p.scale_log2, -lv[jj]));
+                  acc1 += fast_ex2(fmaf(x[jj + 1], p.scale_log2, -lv[jj + 1]));
+                }
               } else {
 #pragma unroll
                 for (int jj = 0; jj < 16; ++jj)
-                  x[jj] = (tvalid && n0 + jj < NV) ? fast_ex2(fmaf(x[jj], p.scale_log2, -lse)) : 0.f;
+                  if (ct + jj < g.NT) acc0 += fast_ex2(fmaf(x[jj], p.scale_log2, -lv[jj]));
               }
             } else {
 #pragma unroll
-              for (int jj = 0; jj < 16; ++jj)
-                x[jj] = (tvalid && n0 + jj < NV) ? x[jj] * p.scale : 0.f;
+              for (int jj = 0; jj < 16; jj += 2) {
+                if (ct + jj < g.NT) acc0 += x[jj];
+                if (ct + jj + 1 < g.NT) acc1 += x[jj + 1];
+              }
             }
-            r = reduce_scatter16(x, lane, AddOp());
+            cp[c * kTileKeys + lrow] = acc0 + acc1;
           }
-          if ((lane & 1) == 0) cp[q4 * kTileKeys + c16 + (lane >> 1)] = r;
         }
         ptx::tc_fence_before();
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(a_empty + buf);
-        ptx::named_bar(2 + cg, 128);   // the four lane quarters of this column group
-        if (q4 % kQph == 0 && hs < g.nh) {
-          const int col = cg * 32 + lane;
-          const int n = kTileKeys * j + col;
+        ptx::named_bar(2 + q4, 128);   // the four column groups of this lane quarter
+        if (cg < g.nh) {
+          const int n = kTileKeys * j + lrow;   // visual index of this lane's key
           if (n < NV) {
-            float a = cp[q4 * kTileKeys + col];
+            const int c0 = cg * kCph;
+            float a = cp[c0 * kTileKeys + lrow];
 #pragma unroll
-            for (int k = 1; k < kQph; ++k) a += cp[(q4 + k) * kTileKeys + col];
-            a *= inv_nt;
-            p.a_out[((size_t)g.l * la.H + g.h + hs) * (size_t)la.sum_vis + g.v0 + n] = a;
+            for (int c = 1; c < kCph; ++c)
+              if (c < head_chunks) a += cp[(c0 + c) * kTileKeys + lrow];
+            a *= a_mul;
+            p.a_out[((size_t)g.l * la.H + g.h + cg) * (size_t)la.sum_vis + g.v0 + n] = a;
             const float al = a * kLog2e, mnew = fmaxf(st_m, al);
             st_e = st_e * fast_ex2(st_m - mnew) + fast_ex2(al - mnew);
             st_m = mnew;
@@ -410,9 +423,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      // ---- statistics of each head's visual scores: merge the 128 producing
-      // lanes of the head (four warps, one per column group) in a fixed order
-      if (q4 % kQph == 0) {
+      // ---- statistics of each head's visual scores: merge the lanes of the
+      // head's four reducing warps (one per lane quarter) in a fixed order
+      if (cg < HPU) {
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
           const float s2 = __shfl_xor_sync(0xffffffffu, st_s, o);
@@ -421,7 +434,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           st_s += s2;
           lse_merge(st_m, st_e, m2, e2);
         }
-        if (lane == 0) red[hs * 4 + cg] = make_float4(st_s, st_m, st_e, 0.f);
+        if (lane == 0) red[cg * 4 + q4] = make_float4(st_s, st_m, st_e, 0.f);
       }
       ptx::named_bar(1, kEpiThreads);
       if (et < g.nh && g.ok) {   // thread et merges stacked head et
@@ -433,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         p.stats[((size_t)g.b * la.L + g.l) * la.H + g.h + et] = stats_entry(S, M, E);
       }
-      // ms, cps and red are rewritten by the next unit only after this barrier
+      // ms, lse_s, cps and red are rewritten by the next unit only after this barrier
       ptx::named_bar(1, kEpiThreads);
     }
   }
