@@ -48,6 +48,8 @@ constexpr int kTileKeys = 128;                // keys per tile (N)
 constexpr int kHalfBytes = 128 * 128;         // 128 rows x 64 bf16
 constexpr int kTileBytes = 2 * kHalfBytes;    // one 128 x 128 bf16 operand
 constexpr int kMaxStages = 8;                 // K ring depth: as many as shared memory holds
+constexpr int kMaxBatch = 8;                  // sweep-2 tiles of a batch unit (whole TMEM)
+constexpr int kTmemCols = 512;                // two 128-column accumulators, or a batch
 constexpr int kEpiWarps = 16;
 constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr int kThreads = 64 + kEpiThreads;
@@ -78,8 +80,8 @@ __host__ __device__ inline SPlan stream_plan(int stages) {
   SPlan s;
   s.q = 0;                                              // [2 halves][128 rows][128 B]
   s.k = (uint32_t)kTileBytes;                           // [stages][tile]
-  s.bars = s.k + (uint32_t)stages * kTileBytes;         // 2 + 2*kMaxStages + 4 mbarriers
-  s.slot = s.bars + 8u * (uint32_t)(2 + 2 * kMaxStages + 4);
+  s.bars = s.k + (uint32_t)stages * kTileBytes;         // mbarriers, see the kernel
+  s.slot = s.bars + 8u * (uint32_t)(2 + 2 * kMaxStages + 4 + kMaxBatch + 1);
   s.ms = (s.slot + 16u + 15u) & ~15u;                   // [4][128] float2 (max, sum)
   s.lse = s.ms + 4u * kRows * 8u;                       // [128] float lse per text row
   s.cps = s.lse + kRows * 4u;                           // [2][8 chunks][128 keys] partials
@@ -88,14 +90,27 @@ __host__ __device__ inline SPlan stream_plan(int stages) {
   return s;
 }
 
+// Text columns of the sweep-2 accumulator: the unit's rows rounded up to the
+// MMA's N granularity (16), or every lane of a stack of heads.
+template <int HPU>
+__device__ __forceinline__ int sweep2_cols(int NT) {
+  return HPU == 1 ? min(kRows, max(16, (NT + 15) & ~15)) : kRows;
+}
+
 // Geometry of one unit, derived identically by every warp role.
 struct SGeo {
   int b, l, h, kvh, nh, S, NV, NT, t0, x0, v0;   // heads h .. h + nh - 1
   int n1, n2;   // key tiles of sweep 1 (whole causal prefix) and sweep 2 (visual)
-  bool ok;
+  // Batch units (causal, one head, every sweep-2 accumulator fits TMEM at
+  // once, every visual tile fits the K ring): sweep 1 takes n_st tiles ending
+  // at key S (keys < 0 masked), the n2 visual tiles from key S and n_tt text
+  // tiles, starting at key kfirst; the visual tiles stay in the ring and
+  // sweep 2 issues all its MMAs at once from there.
+  int n_st, n_tt, kfirst;
+  bool ok, batch;
 };
 
-template <int HPU>
+template <int HPU, bool SPLIT>
 __device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit) {
   const LayoutArgs& la = p.la;
   SGeo g;
@@ -120,27 +135,29 @@ __device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit) {
   g.x0 = __ldg(la.text_off + g.b);
   g.v0 = __ldg(la.vis_off + g.b);
   const int T = g.S + g.NV + g.NT;
-  g.ok = g.S >= 0 && g.NV >= 0 && g.NT >= 1 && g.NT <= kRows / HPU && T <= la.max_T &&
+  g.ok = g.S >= 0 && g.NV >= 0 && g.NT >= 1 && g.NT <= (SPLIT ? kRows / 2 : kRows / HPU) && T <= la.max_T &&
          g.NV <= la.max_vis && __ldg(la.tok_off + g.b + 1) - g.t0 == T && g.t0 >= 0 &&
          g.t0 + T <= la.sum_T && __ldg(la.text_off + g.b + 1) - g.x0 == g.NT && g.x0 >= 0 &&
          g.x0 + g.NT <= la.sum_text && __ldg(la.vis_off + g.b + 1) - g.v0 == g.NV &&
          g.v0 >= 0 && g.v0 + g.NV <= la.sum_vis;
   const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
-  g.n1 = g.ok && causal ? (T + kTileKeys - 1) / kTileKeys : 0;
   g.n2 = g.ok ? (g.NV + kTileKeys - 1) / kTileKeys : 0;
+  g.n_st = (g.S + kTileKeys - 1) / kTileKeys;
+  g.n_tt = max(0, (g.NV + g.NT + kTileKeys - 1) / kTileKeys - g.n2);
+  g.batch = HPU == 1 && g.ok && causal && g.n2 >= 1 && g.n2 <= kMaxBatch &&
+            g.n2 * sweep2_cols<HPU>(g.NT) <= kTmemCols && g.n2 + g.n_tt <= p.stages;
+  g.kfirst = g.batch ? g.S - kTileKeys * g.n_st : 0;
+  g.n1 = !(g.ok && causal) ? 0
+         : g.batch ? g.n_st + g.n2 + g.n_tt : (T + kTileKeys - 1) / kTileKeys;
   return g;
 }
 
-// Text columns of the sweep-2 accumulator: the unit's rows rounded up to the
-// MMA's N granularity (16), or every lane of a stack of heads.
-template <int HPU>
-__device__ __forceinline__ int sweep2_cols(int NT) {
-  return HPU == 1 ? min(kRows, max(16, (NT + 15) & ~15)) : kRows;
-}
-
 // HPU: query heads stacked per unit (1, 2 or 4), fixed at compile time so that
-// the row mapping and the quarter sums are unrolled.
-template <int HPU>
+// the row mapping and the quarter sums are unrolled.  SPLIT (one head of at
+// most 64 text rows): the queries fill TMEM lanes 0-63 and again 64-127, and
+// in sweep 1 each half of the lanes takes half of every key tile's columns, so
+// all four lane quarters (all four SM sub-partitions) share the exponentials.
+template <int HPU, bool SPLIT>
 __global__ void __launch_bounds__(kThreads, 1)
     score_stream_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmK, const StreamArgs p) {
@@ -149,6 +166,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const LayoutArgs& la = p.la;
   const SPlan plan = stream_plan(p.stages);
+  constexpr uint32_t q_half = kHalfBytes;   // bytes of one 64-element half of Q
   uint8_t* q_sm = smem + plan.q;
   uint8_t* k_sm = smem + plan.k;
   uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + plan.bars);
@@ -157,6 +175,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* k_empty = k_full + kMaxStages; // [kMaxStages]
   uint64_t* a_full = k_empty + kMaxStages; // [2] accumulator buffer ready
   uint64_t* a_empty = a_full + 2;          // [2] accumulator buffer read
+  uint64_t* b_full = a_empty + 2;          // [kMaxBatch] batch sweep-2 accumulator ready
+  uint64_t* b_done = b_full + kMaxBatch;   // batch sweep 2 read: TMEM free again
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + plan.slot);
   float2* ms = reinterpret_cast<float2*>(smem + plan.ms);
   float* lse_s = reinterpret_cast<float*>(smem + plan.lse);
@@ -182,12 +202,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::mbar_init(a_full + i, 1);
       ptx::mbar_init(a_empty + i, kEpiWarps);
     }
+    for (int i = 0; i < kMaxBatch; ++i) ptx::mbar_init(b_full + i, 1);
+    ptx::mbar_init(b_done, kEpiWarps);
     ptx::fence_barrier_init();
     ptx::fence_proxy_async_smem();
     ptx::prefetch_tensormap(&tmQ);
     ptx::prefetch_tensormap(&tmK);
   }
-  if (warp == 1) ptx::tmem_alloc(tmem_slot, 256);
+  if (warp == 1) ptx::tmem_alloc(tmem_slot, kTmemCols);
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
@@ -200,7 +222,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       int ld = 0, u = 0;
       for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x, ++u) {
-        const SGeo g = stream_geo<HPU>(p, unit);
+        const SGeo g = stream_geo<HPU, SPLIT>(p, unit);
         if (!g.ok) E2S_DEV_FLAG(p.status, E2S_ERR_SHAPE);
         if (u > 0 && !ptx::mbar_wait(q_empty, (u - 1) & 1, limit, p.status))
           limit = kWaitNsAfterFault;
@@ -208,23 +230,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           // kRows / HPU rows of each stacked head (an absent head repeats the last one;
           // its rows are masked)
           const int qrow = g.l * la.sum_text + g.x0;
-          ptx::mbar_arrive_expect_tx(q_full, (uint32_t)kTileBytes);
+          ptx::mbar_arrive_expect_tx(q_full, 2u * q_half);
 #pragma unroll
-          for (int hs = 0; hs < HPU; ++hs) {
-            const int hq = g.h + min(hs, g.nh - 1);
-            const uint32_t off = (uint32_t)(hs * kRph) * 128u;
+          for (int hs = 0; hs < (SPLIT ? 2 : HPU); ++hs) {
+            const int hq = SPLIT ? g.h : g.h + min(hs, g.nh - 1);
+            const uint32_t off = (uint32_t)(hs * (SPLIT ? kRows / 2 : kRph)) * 128u;
             ptx::tma_load_3d(q_sm + off, &tmQ, q_full, 0, hq, qrow);
-            ptx::tma_load_3d(q_sm + kHalfBytes + off, &tmQ, q_full, 64, hq, qrow);
+            ptx::tma_load_3d(q_sm + q_half + off, &tmQ, q_full, 64, hq, qrow);
           }
         } else {
           ptx::mbar_arrive(q_full);
         }
-        for (int j = 0; j < g.n1 + g.n2; ++j, ++ld) {
+        // sweep-1 tiles, then (except in a batch unit, whose visual tiles stay
+        // in the ring) the visual tiles again for sweep 2
+        for (int j = 0; j < g.n1 + (g.batch ? 0 : g.n2); ++j, ++ld) {
           const int s = ld % p.stages;
           if (ld >= p.stages &&
               !ptx::mbar_wait(k_empty + s, (ld / p.stages - 1) & 1, limit, p.status))
             limit = kWaitNsAfterFault;
-          const int key0 = j < g.n1 ? kTileKeys * j : g.S + kTileKeys * (j - g.n1);
+          const int key0 = j < g.n1 ? g.kfirst + kTileKeys * j : g.S + kTileKeys * (j - g.n1);
           const int krow = g.l * la.sum_T + g.t0 + key0;
           ptx::mbar_arrive_expect_tx(k_full + s, (uint32_t)kTileBytes);
           ptx::tma_load_3d(k_sm + s * kTileBytes, &tmK, k_full + s, 0, g.kvh, krow);
@@ -238,12 +262,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       const uint32_t idesc1 = ptx::idesc_bf16_f32(kRows, kTileKeys);
       const uint32_t q_base = ptx::smem_addr(q_sm);
-      int ld = 0, tc = 0, u = 0;
+      int ld = 0, tc = 0, u = 0, bu = 0;
+      auto mma_tile = [&](uint32_t d, uint32_t a_base, uint32_t a_half, uint32_t b_base,
+                          uint32_t b_half, uint32_t idesc) {
+#pragma unroll
+        for (int ks = 0; ks < 8; ++ks) {
+          const uint32_t half = ks >> 2, kk = ks & 3;
+          const uint64_t ad = ptx::sdesc_sw128(a_base + half * a_half + kk * 32u);
+          const uint64_t bd = ptx::sdesc_sw128(b_base + half * b_half + kk * 32u);
+          ptx::mma_bf16(d, ad, bd, idesc, ks > 0 ? 1u : 0u);
+        }
+      };
       for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x, ++u) {
-        const SGeo g = stream_geo<HPU>(p, unit);
-        const uint32_t idesc2 = ptx::idesc_bf16_f32(kTileKeys, sweep2_cols<HPU>(g.NT));
+        const SGeo g = stream_geo<HPU, SPLIT>(p, unit);
+        const int n2c = sweep2_cols<HPU>(g.NT);
+        const uint32_t idesc2 = ptx::idesc_bf16_f32(kTileKeys, n2c);
         if (!ptx::mbar_wait(q_full, u & 1, limit, p.status)) limit = kWaitNsAfterFault;
-        for (int j = 0; j < g.n1 + g.n2; ++j, ++ld, ++tc) {
+        const int ld_vis = ld + g.n_st;   // load index of a batch unit's first visual tile
+        for (int j = 0; j < g.n1 + (g.batch ? 0 : g.n2); ++j, ++ld, ++tc) {
           const int s = ld % p.stages, buf = tc & 1;
           if (!ptx::mbar_wait(k_full + s, (ld / p.stages) & 1, limit, p.status))
             limit = kWaitNsAfterFault;
@@ -251,21 +287,41 @@ __global__ void __launch_bounds__(kThreads, 1)
             limit = kWaitNsAfterFault;
           ptx::tc_fence_after();
           const uint32_t k_base = ptx::smem_addr(k_sm + s * kTileBytes);
-          const bool sw2 = j >= g.n1;
-          const uint32_t a_base = sw2 ? k_base : q_base, b_base = sw2 ? q_base : k_base;
-          const uint32_t idesc = sw2 ? idesc2 : idesc1;
           const uint32_t d = tmem + (uint32_t)(buf * kTileKeys);
-#pragma unroll
-          for (int ks = 0; ks < 8; ++ks) {
-            const uint32_t half = ks >> 2, kk = ks & 3;
-            const uint64_t ad = ptx::sdesc_sw128(a_base + half * kHalfBytes + kk * 32u);
-            const uint64_t bd = ptx::sdesc_sw128(b_base + half * kHalfBytes + kk * 32u);
-            ptx::mma_bf16(d, ad, bd, idesc, ks > 0 ? 1u : 0u);
-          }
-          ptx::mma_commit(k_empty + s);   // the producer may refill the stage
+          if (j >= g.n1)
+            mma_tile(d, k_base, kHalfBytes, q_base, q_half, idesc2);
+          else
+            mma_tile(d, q_base, q_half, k_base, kHalfBytes, idesc1);
+          const int vi = j - g.n_st;   // a batch unit keeps its visual tiles
+          if (!(g.batch && vi >= 0 && vi < g.n2)) ptx::mma_commit(k_empty + s);
           ptx::mma_commit(a_full + buf);  // the epilogue may read the buffer
         }
+        if (g.batch) {
+          // every sweep-1 accumulator read: the sweep-2 accumulators of all
+          // visual tiles go side by side into TMEM columns j * n2c
+          for (int k = 1; k <= 2; ++k) {
+            const int tp = tc - k;
+            if (tp >= 0 && !ptx::mbar_wait(a_empty + (tp & 1), (tp / 2) & 1, limit, p.status))
+              limit = kWaitNsAfterFault;
+          }
+          ptx::tc_fence_after();
+          for (int j = 0; j < kMaxBatch; ++j) {
+            if (j < g.n2) {
+              const int s = (ld_vis + j) % p.stages;
+              mma_tile(tmem + (uint32_t)(j * n2c), ptx::smem_addr(k_sm + s * kTileBytes),
+                       kHalfBytes, q_base, q_half, idesc2);
+              ptx::mma_commit(k_empty + s);
+              ptx::mma_commit(b_full + j);
+            } else {
+              ptx::mbar_arrive(b_full + j);   // keep every barrier's phase in step
+            }
+          }
+        }
         ptx::mma_commit(q_empty);   // every MMA of the unit is done with Q
+        if (g.batch) {   // the next unit's accumulators wait for the batch to be read
+          if (!ptx::mbar_wait(b_done, bu & 1, limit, p.status)) limit = kWaitNsAfterFault;
+          ++bu;
+        }
       }
     }
   } else {
@@ -276,12 +332,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int lrow = q4 * 32 + lane;         // this lane's TMEM row
     const uint32_t lane_base = (uint32_t)(q4 * 32) << 16;
     const int et = threadIdx.x - 64;
-    int tc = 0;
+    int tc = 0, bu = 0;
     for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x) {
-      const SGeo g = stream_geo<HPU>(p, unit);
-      // TMEM row lrow holds text row t of stacked head hs
-      const int hs = lrow / kRph, t = lrow - hs * kRph;
-      const bool rows_live = hs < g.nh && (q4 * 32) % kRph < g.NT;   // warp-uniform
+      const SGeo g = stream_geo<HPU, SPLIT>(p, unit);
+      // TMEM row lrow holds text row t of stacked head hs (SPLIT: row lrow % 64)
+      const int hs = SPLIT ? 0 : lrow / kRph;
+      const int t = SPLIT ? (lrow & (kRows / 2 - 1)) : lrow - hs * kRph;
+      const bool rows_live =
+          hs < g.nh && (SPLIT ? (q4 & 1) * 32 : (q4 * 32) % kRph) < g.NT;   // warp-uniform
       const bool tvalid = hs < g.nh && t < g.NT;
       const int lim = tvalid ? g.S + g.NV + t : -1;   // last key this row sees
       const float inv_nt = 1.f / (float)max(g.NT, 1);
@@ -294,12 +352,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tc_fence_after();
         if (rows_live) {
 #pragma unroll
-          for (int ch = 0; ch < 2; ++ch) {
-            const int c16 = cg * 32 + ch * 16;
-            const int key0 = kTileKeys * j + c16;
+          for (int ch = 0; ch < (SPLIT ? 1 : 2); ++ch) {
+            // 16-column chunks of this warp: 2 of its column group's 32, or
+            // (SPLIT) 1 of the 64 columns of its lane half
+            const int c16 = SPLIT ? (q4 >> 1) * (kTileKeys / 2) + cg * 16 : cg * 32 + ch * 16;
+            const int key0 = g.kfirst + kTileKeys * j + c16;
             float x[16];
             ptx::tmem_ld16(tmem + lane_base + (uint32_t)(buf * kTileKeys + c16), x);
-            if (key0 + 15 <= lim) {   // the row sees the whole chunk
+            if (key0 >= 0 && key0 + 15 <= lim) {   // the row sees the whole chunk
               float cmax = x[0];
 #pragma unroll
               for (int jj = 1; jj < 16; ++jj) cmax = fmaxf(cmax, x[jj]);
@@ -312,16 +372,17 @@ __global__ void __launch_bounds__(kThreads, 1)
               }
               ssum = acc0 + acc1;
               m = mnew;
-            } else if (key0 <= lim) {   // the chunk straddles the row's last key
+            } else if (key0 <= lim && key0 + 15 >= 0) {   // key 0 or the row's last key inside
               float cmax = kNegBig;
 #pragma unroll
               for (int jj = 0; jj < 16; ++jj)
-                if (key0 + jj <= lim) cmax = fmaxf(cmax, x[jj]);
+                if (key0 + jj >= 0 && key0 + jj <= lim) cmax = fmaxf(cmax, x[jj]);
               const float mnew = fmaxf(m, cmax * p.scale_log2);
               float acc = ssum * fast_ex2(m - mnew);
 #pragma unroll
               for (int jj = 0; jj < 16; ++jj)
-                if (key0 + jj <= lim) acc += fast_ex2(fmaf(x[jj], p.scale_log2, -mnew));
+                if (key0 + jj >= 0 && key0 + jj <= lim)
+                  acc += fast_ex2(fmaf(x[jj], p.scale_log2, -mnew));
               ssum = acc;
               m = mnew;
             }
@@ -336,16 +397,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (causal) {
         ms[cg * kRows + lrow] = make_float2(m, ssum);
         ptx::named_bar(1, kEpiThreads);
+        // partials of this row: four column groups (and, SPLIT, both lane halves)
+        constexpr int kParts = SPLIT ? 8 : 4;
+        auto part = [&](int c) {
+          return ms[(c & 3) * kRows + (c < 4 ? lrow : (lrow ^ (kRows / 2)))];
+        };
         float M = kNegBig;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) M = fmaxf(M, ms[c * kRows + lrow].x);
+        for (int c = 0; c < kParts; ++c) M = fmaxf(M, part(c).x);
         float L = 0.f;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const float2 v = ms[c * kRows + lrow];
+        for (int c = 0; c < kParts; ++c) {
+          const float2 v = part(c);
           L += v.y * fast_ex2(v.x - M);
         }
-        if (cg == 0) lse_s[lrow] = L > 0.f ? M + __log2f(L) : kNegBig;
+        if (cg == 0 && (!SPLIT || lrow < kRows / 2)) lse_s[lrow] = L > 0.f ? M + __log2f(L) : kNegBig;
         ptx::named_bar(1, kEpiThreads);
       }
       // ---- sweep 2: accumulator D[key][column], keys on the lanes, so each
@@ -360,6 +426,59 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int head_chunks = min(kCph, (g.NT + 15) >> 4);
       const float a_mul = causal ? inv_nt : p.scale * inv_nt;
       float st_s = 0.f, st_m = kNegBig, st_e = 0.f;
+      if (g.batch) {
+        // batch unit: the accumulator of visual tile j sits in columns
+        // j * 16 * nch; column group cg owns the tiles j % 4 == cg and sums
+        // every column of its lanes' keys -- no cross-warp reduction
+        for (int j = cg; j < g.n2; j += 4) {
+          if (!ptx::mbar_wait(b_full + j, bu & 1, limit, p.status)) limit = kWaitNsAfterFault;
+          ptx::tc_fence_after();
+          const int n = kTileKeys * j + lrow;   // visual index of this lane's key
+          float a = 0.f;
+          if (kTileKeys * j + q4 * 32 < NV) {   // the warp holds visual keys
+            const uint32_t tb = tmem + lane_base + (uint32_t)(j * nch * 16);
+            for (int c = 0; c < nch; ++c) {
+              float x[16];
+              ptx::tmem_ld16(tb + (uint32_t)(c * 16), x);
+              const float4* l4 = reinterpret_cast<const float4*>(lse_s + c * 16);
+              float s0 = 0.f, s1 = 0.f;
+              if (c * 16 + 15 < g.NT) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                  const float4 v = l4[q];
+                  s0 += fast_ex2(fmaf(x[4 * q], p.scale_log2, -v.x));
+                  s1 += fast_ex2(fmaf(x[4 * q + 1], p.scale_log2, -v.y));
+                  s0 += fast_ex2(fmaf(x[4 * q + 2], p.scale_log2, -v.z));
+                  s1 += fast_ex2(fmaf(x[4 * q + 3], p.scale_log2, -v.w));
+                }
+              } else {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                  const float4 v = l4[q];
+                  const float lv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                  for (int i = 0; i < 4; ++i)
+                    if (c * 16 + 4 * q + i < g.NT)
+                      s0 += fast_ex2(fmaf(x[4 * q + i], p.scale_log2, -lv[i]));
+                }
+              }
+              a += s0 + s1;
+            }
+          }
+          if (n < NV) {
+            a *= a_mul;
+            p.a_out[((size_t)g.l * la.H + g.h) * (size_t)la.sum_vis + g.v0 + n] = a;
+            const float al = a * kLog2e, mnew = fmaxf(st_m, al);
+            st_e = st_e * fast_ex2(st_m - mnew) + fast_ex2(al - mnew);
+            st_m = mnew;
+            st_s += a;
+          }
+        }
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(b_done);
+        ++bu;
+      } else
       for (int j = 0; j < g.n2; ++j, ++tc) {
         const int buf = tc & 1;
         float* cp = cps + (j & 1) * 8 * kTileKeys;
@@ -424,8 +543,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       // ---- statistics of each head's visual scores: merge the lanes of the
-      // head's four reducing warps (one per lane quarter) in a fixed order
-      if (cg < HPU) {
+      // head's reducing warps (one per lane quarter; in a batch unit all 16)
+      // in a fixed order
+      if (g.batch || cg < HPU) {
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
           const float s2 = __shfl_xor_sync(0xffffffffu, st_s, o);
@@ -434,12 +554,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           st_s += s2;
           lse_merge(st_m, st_e, m2, e2);
         }
-        if (lane == 0) red[cg * 4 + q4] = make_float4(st_s, st_m, st_e, 0.f);
+        if (lane == 0) red[g.batch ? ew : cg * 4 + q4] = make_float4(st_s, st_m, st_e, 0.f);
       }
       ptx::named_bar(1, kEpiThreads);
       if (et < g.nh && g.ok) {   // thread et merges stacked head et
         float S = 0.f, M = kNegBig, E = 0.f;
-        for (int c = 0; c < 4; ++c) {
+        const int nr = g.batch ? kEpiWarps : 4;
+        for (int c = 0; c < nr; ++c) {
           const float4 r4 = red[et * 4 + c];
           S += r4.x;
           lse_merge(M, E, r4.y, r4.z);
@@ -455,7 +576,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (warp == 1) {
     ptx::tc_fence_after();
-    ptx::tmem_dealloc(tmem, 256);
+    ptx::tmem_dealloc(tmem, kTmemCols);
   }
 }
 
@@ -482,12 +603,12 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
   StreamArgs p;
   p.la = la;
   p.mode = mode;
-  p.stages = stream_stages();
   p.group = la.H / la.H_kv;
   // stack the query heads of one kv head into the 128 TMEM lanes when their
   // text rows leave room (64 rows: two heads, 32 rows: four)
   int hpu = 1;
   while (hpu < 4 && hpu * 2 <= p.group && la.max_text <= kRows / (hpu * 2)) hpu *= 2;
+  p.stages = stream_stages();
   p.upk = (p.group + hpu - 1) / hpu;
   p.num_units = la.B * la.L * la.H_kv * p.upk;
   p.scale = 1.0f / sqrtf(128.0f);
@@ -498,20 +619,26 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
   p.status = status;
   if (p.num_units == 0 || la.sum_vis == 0) return cudaSuccess;
   CUtensorMap tmQ, tmK;
-  if (!make_score_map(&tmQ, q, la.H, (int64_t)la.L * la.sum_text, q_stride, kRows / hpu) ||
+  // one head of at most 64 text rows: the queries are loaded twice (SPLIT)
+  const bool split = hpu == 1 && la.max_text <= kRows / 2;
+  if (!make_score_map(&tmQ, q, la.H, (int64_t)la.L * la.sum_text, q_stride,
+                      split ? kRows / 2 : kRows / hpu) ||
       !make_score_map(&tmK, k, la.H_kv, (int64_t)la.L * la.sum_T, k_stride, kTileKeys))
     return cudaErrorInvalidValue;
   if (p.stages < 2) return cudaErrorInvalidValue;
   const size_t smem = stream_plan(p.stages).total + 1024;
   const dim3 grid((unsigned)std::min(p.num_units, sm_count()));
   if (hpu == 4)
-    return launch_kernel(score_stream_kernel<4>, grid, dim3(kThreads), smem, st, 0, false, tmQ,
-                         tmK, p);
+    return launch_kernel(score_stream_kernel<4, false>, grid, dim3(kThreads), smem, st, 0, false,
+                         tmQ, tmK, p);
   if (hpu == 2)
-    return launch_kernel(score_stream_kernel<2>, grid, dim3(kThreads), smem, st, 0, false, tmQ,
-                         tmK, p);
-  return launch_kernel(score_stream_kernel<1>, grid, dim3(kThreads), smem, st, 0, false, tmQ, tmK,
-                       p);
+    return launch_kernel(score_stream_kernel<2, false>, grid, dim3(kThreads), smem, st, 0, false,
+                         tmQ, tmK, p);
+  if (split)
+    return launch_kernel(score_stream_kernel<1, true>, grid, dim3(kThreads), smem, st, 0, false,
+                         tmQ, tmK, p);
+  return launch_kernel(score_stream_kernel<1, false>, grid, dim3(kThreads), smem, st, 0, false,
+                       tmQ, tmK, p);
 }
 
 }  // namespace e2s

@@ -62,10 +62,11 @@ __device__ __forceinline__ bool mbar_try_wait_hint(uint64_t* bar, uint32_t parit
 }
 
 // Waits for phase `parity` of `bar` for at most `limit_ns`.  Returns false
-// (and records E2S_ERR_TIMEOUT in *status) if the limit ran out.
-static __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns,
-                                       uint32_t* status) {
-  if (mbar_try_wait(bar, parity)) return true;
+// (and records E2S_ERR_TIMEOUT in *status) if the limit ran out.  The check of
+// an already completed phase is inline; only the bounded polling loop is a
+// call (a call costs hundreds of cycles in saved registers).
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity,
+                                                   uint64_t limit_ns, uint32_t* status) {
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t it = 0;; ++it) {
     if (mbar_try_wait_hint(bar, parity, 20000u)) return true;
@@ -74,6 +75,10 @@ static __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, ui
       return false;
     }
   }
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns,
+                                          uint32_t* status) {
+  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, limit_ns, status);
 }
 
 // ---------------------------------------------------------------- TMA
