@@ -41,28 +41,32 @@ UNIT = "images/s"
 # workload; the others exist for profiling and context lines.
 WORKLOADS = {
     "cfg1": (1, 64, None, "llava-1.5-7b decision+compaction, batch 1, 35+576(24x24)+64 tokens, "
-                          "3 layers, 32x128 MHA, K=64 (configs[1])"),
+                          "3 layers, 32x128 MHA, K=64"),
     "cfg2": (2, 64, None, "llava-1.5-7b decision+compaction, batch 32, 35+576(24x24)+U[16,128] "
-                          "ragged text tokens, 3 layers, 32x128 MHA, K=64 (configs[2])"),
+                          "ragged text tokens, 3 layers, 32x128 MHA, K=64"),
     "cfg3": (3, None, None, "qwen2-vl-7b decision+compaction, batch 16, grids 16x16..36x36, "
-                            "28q/4kv heads, 3 layers, K=11.1% (configs[3])"),
+                            "28q/4kv heads, 3 layers, K=11.1%"),
     "cfg4": (4, None, None, "high-res decision+compaction, batch 8, 48x48/64x64 grids, 128 text, "
-                            "4 layers, 32x128 MHA, K=11% (configs[4])"),
+                            "4 layers, 32x128 MHA, K=11%"),
 }
 
 # ncu dram__bytes_read.sum + dram__bytes_write.sum of one launch of the dominant
-# kernel on a workload (ncu --set full, its default cache control: cold caches),
-# with the sha256 (first 16 hex) of the kernel's source when it was captured; a
-# source that has changed since reports null traffic.
+# kernel on a workload (ncu's default cache control: cold caches), with the
+# sha256 (first 16 hex) of the kernel's sources (its .cu and the device headers
+# it includes) when it was captured; sources that have changed since report
+# null traffic.
+KERNEL_SOURCES = ("score_unit.cu", "sm100_ptx.cuh", "device_common.cuh")
 NCU_TRAFFIC = {
-    "cfg1": {"stage": "score", "kernel": "score_unit_kernel", "src": "score_unit.cu",
-             "sha": "7adc1246b14580db", "bytes": 18220000},
+    "cfg1": {"stage": "score", "kernel": "score_unit_kernel", "src": KERNEL_SOURCES,
+             "sha": "38ec279d0f5f240c", "bytes": 18230000},
 }
 
 
-def _src_hash(name: str) -> str:
-    p = os.path.join(ROOT, "paper_2608_23253_gb300", "csrc", name)
-    return hashlib.sha256(open(p, "rb").read()).hexdigest()[:16]
+def _src_hash(names) -> str:
+    h = hashlib.sha256()
+    for name in names:
+        h.update(open(os.path.join(ROOT, "paper_2608_23253_gb300", "csrc", name), "rb").read())
+    return h.hexdigest()[:16]
 
 
 def combine_ranks(total_ms: float, e2e_ms: float, images_per_rank: int, world: int, device):
