@@ -262,15 +262,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       const uint32_t idesc1 = ptx::idesc_bf16_f32(kRows, kTileKeys);
       const uint32_t q_base = ptx::smem_addr(q_sm);
-      int ld = 0, tc = 0, u = 0, bu = 0;
-      auto mma_tile = [&](uint32_t d, uint32_t a_base, uint32_t a_half, uint32_t b_base,
-                          uint32_t b_half, uint32_t idesc) {
+      int tc = 0, u = 0, bu = 0;
+      int slot = 0;          // ring stage of the next tile to consume
+      uint32_t kph = 0u;     // its k_full phase
+      // both operands are two 64-element halves of 128 rows (kHalfBytes apart)
+      auto mma_tile = [&](uint32_t d, uint32_t a_base, uint32_t b_base, uint32_t idesc) {
+        // one descriptor per operand; each K step of 16 adds its byte offset
+        // (>> 4) to the 14-bit start-address field, which cannot carry for
+        // shared-memory addresses below 256 KiB
+        const uint64_t a0 = ptx::sdesc_sw128(a_base), b0 = ptx::sdesc_sw128(b_base);
 #pragma unroll
         for (int ks = 0; ks < 8; ++ks) {
           const uint32_t half = ks >> 2, kk = ks & 3;
-          const uint64_t ad = ptx::sdesc_sw128(a_base + half * a_half + kk * 32u);
-          const uint64_t bd = ptx::sdesc_sw128(b_base + half * b_half + kk * 32u);
-          ptx::mma_bf16(d, ad, bd, idesc, ks > 0 ? 1u : 0u);
+          const uint32_t off = (half * (uint32_t)kHalfBytes + kk * 32u) >> 4;
+          ptx::mma_bf16(d, a0 + off, b0 + off, idesc, ks > 0 ? 1u : 0u);
         }
       };
       for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x, ++u) {
@@ -278,20 +283,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int n2c = sweep2_cols<HPU>(g.NT);
         const uint32_t idesc2 = ptx::idesc_bf16_f32(kTileKeys, n2c);
         if (!ptx::mbar_wait(q_full, u & 1, limit, p.status)) limit = kWaitNsAfterFault;
-        const int ld_vis = ld + g.n_st;   // load index of a batch unit's first visual tile
-        for (int j = 0; j < g.n1 + (g.batch ? 0 : g.n2); ++j, ++ld, ++tc) {
-          const int s = ld % p.stages, buf = tc & 1;
-          if (!ptx::mbar_wait(k_full + s, (ld / p.stages) & 1, limit, p.status))
-            limit = kWaitNsAfterFault;
+        const int slot_vis = (slot + g.n_st) % p.stages;   // a batch unit's first visual tile
+        for (int j = 0; j < g.n1 + (g.batch ? 0 : g.n2); ++j, ++tc) {
+          const int s = slot, buf = tc & 1;
+          if (!ptx::mbar_wait(k_full + s, kph, limit, p.status)) limit = kWaitNsAfterFault;
+          if (++slot == p.stages) {
+            slot = 0;
+            kph ^= 1u;
+          }
           if (tc >= 2 && !ptx::mbar_wait(a_empty + buf, (tc / 2 - 1) & 1, limit, p.status))
             limit = kWaitNsAfterFault;
           ptx::tc_fence_after();
           const uint32_t k_base = ptx::smem_addr(k_sm + s * kTileBytes);
           const uint32_t d = tmem + (uint32_t)(buf * kTileKeys);
           if (j >= g.n1)
-            mma_tile(d, k_base, kHalfBytes, q_base, q_half, idesc2);
+            mma_tile(d, k_base, q_base, idesc2);
           else
-            mma_tile(d, q_base, q_half, k_base, kHalfBytes, idesc1);
+            mma_tile(d, q_base, k_base, idesc1);
           const int vi = j - g.n_st;   // a batch unit keeps its visual tiles
           if (!(g.batch && vi >= 0 && vi < g.n2)) ptx::mma_commit(k_empty + s);
           ptx::mma_commit(a_full + buf);  // the epilogue may read the buffer
@@ -307,9 +315,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           ptx::tc_fence_after();
           for (int j = 0; j < kMaxBatch; ++j) {
             if (j < g.n2) {
-              const int s = (ld_vis + j) % p.stages;
-              mma_tile(tmem + (uint32_t)(j * n2c), ptx::smem_addr(k_sm + s * kTileBytes),
-                       kHalfBytes, q_base, q_half, idesc2);
+              const int s = (slot_vis + j) % p.stages;
+              mma_tile(tmem + (uint32_t)(j * n2c), ptx::smem_addr(k_sm + s * kTileBytes), q_base,
+                       idesc2);
               ptx::mma_commit(k_empty + s);
               ptx::mma_commit(b_full + j);
             } else {
