@@ -254,6 +254,29 @@ __global__ void __launch_bounds__(kThreads, 1)
           ptx::tma_load_3d(k_sm + s * kTileBytes, &tmK, k_full + s, 0, g.kvh, krow);
           ptx::tma_load_3d(k_sm + s * kTileBytes + kHalfBytes, &tmK, k_full + s, 64, g.kvh, krow);
         }
+        // every load of this unit issued: the next unit's queries and first key
+        // tiles go to L2, so that its loads do not start from DRAM when this
+        // unit's last MMAs retire
+        const int next = unit + (int)gridDim.x;
+        if (next < p.num_units) {
+          const SGeo gn = stream_geo<HPU, SPLIT>(p, next);
+          if (gn.n1 + gn.n2 > 0) {
+            const int qrow = gn.l * la.sum_text + gn.x0;
+#pragma unroll
+            for (int hs = 0; hs < (SPLIT ? 1 : HPU); ++hs) {
+              const int hq = gn.h + min(hs, gn.nh - 1);
+              ptx::tma_prefetch_3d(&tmQ, 0, hq, qrow);
+              ptx::tma_prefetch_3d(&tmQ, 64, hq, qrow);
+            }
+            const int nt = min(gn.n1 + gn.n2, p.stages);
+            for (int j = 0; j < nt; ++j) {
+              const int key0 = j < gn.n1 ? gn.kfirst + kTileKeys * j : gn.S + kTileKeys * (j - gn.n1);
+              const int krow = gn.l * la.sum_T + gn.t0 + key0;
+              ptx::tma_prefetch_3d(&tmK, 0, gn.kvh, krow);
+              ptx::tma_prefetch_3d(&tmK, 64, gn.kvh, krow);
+            }
+          }
+        }
       }
     }
   } else if (warp == 1) {
