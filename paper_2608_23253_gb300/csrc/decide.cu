@@ -115,9 +115,21 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const DecArgs p) {
   for (int i = tid; i < L * H * 4; i += kDecThreads)
     ptx::cp_async4(reinterpret_cast<float*>(st_s) + i,
                    reinterpret_cast<const float*>(p.stats + (size_t)b * L * H) + i);
-  for (int idx = tid; idx < L * H * kTok; idx += kDecThreads) {
-    const int jj = idx & (kTok - 1), lh = idx >> 6;
-    if (jj < ntok) ptx::cp_async4(A + lh * kRow + jj, p.a + (size_t)lh * plane + v0 + n0 + jj);
+  if (((v0 + n0) & 3) == 0 && (plane & 3) == 0 &&
+      (reinterpret_cast<uintptr_t>(p.a) & 15) == 0) {   // 16-byte copies (4 tokens each)
+    for (int idx = tid; idx < L * H * (kTok / 4); idx += kDecThreads) {
+      const int jj = (idx & (kTok / 4 - 1)) * 4, lh = idx / (kTok / 4);
+      const float* src = p.a + (size_t)lh * plane + v0 + n0 + jj;
+      if (jj + 3 < ntok)
+        ptx::cp_async16(A + lh * kRow + jj, src);
+      else
+        for (int t = jj; t < ntok; ++t) ptx::cp_async4(A + lh * kRow + t, src + (t - jj));
+    }
+  } else {
+    for (int idx = tid; idx < L * H * kTok; idx += kDecThreads) {
+      const int jj = idx & (kTok - 1), lh = idx >> 6;
+      if (jj < ntok) ptx::cp_async4(A + lh * kRow + jj, p.a + (size_t)lh * plane + v0 + n0 + jj);
+    }
   }
   ptx::cp_async_wait_all();
   __syncthreads();
@@ -227,7 +239,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const DecArgs p) {
     return;
   }
   const float lam = (p.flags & (E2S_NO_NOVELTY | E2S_VANILLA)) ? 0.f : p.lam;
-  select_image_from_cells(p.q_out + v0, p.cand ? p.cand + v0 : nullptr, NV, gh, gw, G, lam,
+  select_image_from_cells(p.q_out + v0, p.cand ? p.cand + v0 : nullptr, NV, cells, lam,
                           __ldg(p.keep_count + b), cells_g, reinterpret_cast<uint32_t*>(A),
                           reinterpret_cast<uint8_t*>(A) + 4 * (size_t)la.max_vis, ss,
                           p.q_tilde ? p.q_tilde + v0 : nullptr,

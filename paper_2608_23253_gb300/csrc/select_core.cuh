@@ -258,15 +258,15 @@ static __device__ void select_image(const float* q, const int32_t* cand, int NV,
 
 // The same select for a CTA that did not compute q: the cell arg-max keys
 // (Eqs. 20-21) were reduced into cell_best_g[0 .. G*G) in global memory by the
-// CTAs that did, and q[] was written by them.  This CTA reads the keys (and
+// CTAs that did, and q[] was written by them; cm is the image's cell grid.  This CTA reads the keys (and
 // resets them to zero for the next use) in the same phase as q, then runs
 // steps 2-4.  keys (NV words) and cells (NV bytes) are shared scratch.
 static __device__ void select_image_from_cells(const float* q, const int32_t* cand, int NV,
-                                               int gh, int gw, int G, float lam, int K,
+                                               const CellMap& cm, float lam, int K,
                                                unsigned long long* cell_best_g, uint32_t* keys,
                                                uint8_t* cells, SelectSmem& ss, float* q_tilde,
                                                int32_t* keep, uint32_t* status) {
-  const CellMap cm(gh, gw, G);
+  const int G = cm.G;
   for (int i = threadIdx.x; i < G * G; i += blockDim.x) {
     ss.cell_best[i] = __ldcg(cell_best_g + i);
     cell_best_g[i] = 0ull;
