@@ -97,6 +97,28 @@ def test_gqa_stacked_heads(mode, H, H_kv, texts):
     _check(inp, run_gpu(inp, mode), run_oracle(inp, mode))
 
 
+@pytest.mark.parametrize("mode", ["causal", "eq1"])
+def test_split_rows_long_sequences(mode):
+    """Multi-head attention with at most 64 text rows on sequences too long for
+    the resident-K kernel: the streaming kernel loads the queries into both
+    halves of the accumulator lanes and splits each key tile between them."""
+    ims = [ImageSpec(35, 32, 32, 64, 50, 3, 114), ImageSpec(35, 24, 40, 40, 30, 2, 96),
+           ImageSpec(0, 30, 30, 1, 20, 0, 90)]
+    inp = synth.make_inputs(_spec(ims, L=2, H=8, H_kv=8, cfg_id=97), with_payload=False)
+    _check(inp, run_gpu(inp, mode), run_oracle(inp, mode))
+
+
+@pytest.mark.parametrize("mode", ["causal", "eq1"])
+def test_gqa_batch_units(mode):
+    """Grouped-query heads with 65..128 text rows (no stacking) on small grids:
+    every sweep-2 accumulator of a unit fits TMEM at once (batch units), next to
+    units that stream sweep 2."""
+    ims = [ImageSpec(35, 16, 16, 100, 20, 3, 28), ImageSpec(3, 8, 20, 128, 10, 2, 16),
+           ImageSpec(35, 24, 32, 80, 50, 3, 85)]
+    inp = synth.make_inputs(_spec(ims, L=2, H=14, H_kv=2, cfg_id=98), with_payload=False)
+    _check(inp, run_gpu(inp, mode), run_oracle(inp, mode))
+
+
 def test_all_equal_scores_tie_break():
     """Zero queries give equal logits everywhere: ties resolve to the lower index."""
     inp = config_inputs(0, None, None)
