@@ -26,9 +26,10 @@
 // is double-buffered in TMEM (MMA warp), so loads, MMAs and the epilogue of
 // consecutive tiles overlap.
 //
-// Warp roles (576 threads): warp 0 TMA producer, warp 1 TMEM allocator and MMA
-// issuer, warps 2-17 epilogue: warp w reads TMEM lane quarter w % 4 and column
-// group (w - 2) / 4 (32 keys of each tile in sweep 1, column chunks in sweep 2).
+// Warp roles (608 threads): warp 0 TMA producer, warp 1 TMEM allocator and MMA
+// issuer of the even tiles, warp 18 MMA issuer of the odd tiles, warps 2-17
+// epilogue: warp w reads TMEM lane quarter w % 4 and column group (w - 2) / 4
+// (32 keys of each tile in sweep 1, column chunks in sweep 2).
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -52,7 +53,8 @@ constexpr int kMaxBatch = 8;                  // sweep-2 tiles of a batch unit (
 constexpr int kTmemCols = 512;                // two 128-column accumulators, or a batch
 constexpr int kEpiWarps = 16;
 constexpr int kEpiThreads = 32 * kEpiWarps;
-constexpr int kThreads = 64 + kEpiThreads;
+constexpr int kMmaWarp1 = 2 + kEpiWarps;      // the second MMA issuer (odd tiles)
+constexpr int kThreads = 64 + kEpiThreads + 32;
 constexpr uint64_t kWaitNs = 1000000000ull;
 constexpr uint64_t kWaitNsAfterFault = 1000000ull;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -193,7 +195,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0 && lane == 0) {
     ptx::mbar_init(q_full, 1);
-    ptx::mbar_init(q_empty, 1);
+    ptx::mbar_init(q_empty, 2);   // one commit per MMA issuer
     for (int i = 0; i < kMaxStages; ++i) {
       ptx::mbar_init(k_full + i, 1);
       ptx::mbar_init(k_empty + i, 1);
@@ -279,9 +281,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-  } else if (warp == 1) {
-    // ================= MMA issuer into accumulator buffer tc % 2: sweep 1
-    // D[t][key] (text rows on the lanes), sweep 2 D[key][t] (keys on the lanes)
+  } else if (warp == 1 || warp == kMmaWarp1) {
+    // ================= MMA issuers: sweep 1 D[t][key] (text rows on the
+    // lanes), sweep 2 D[key][t] (keys on the lanes).  Two threads alternate
+    // tiles -- issuer m owns accumulator buffer m and the tiles tc % 2 == m --
+    // so that one's waits and commits overlap the other's MMAs (an issuing
+    // thread is held while the tensor pipe takes its instructions).
+    const int mid = warp == 1 ? 0 : 1;
     if (lane == 0) {
       const uint32_t idesc1 = ptx::idesc_bf16_f32(kRows, kTileKeys);
       const uint32_t q_base = ptx::smem_addr(q_sm);
@@ -309,11 +315,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int slot_vis = (slot + g.n_st) % p.stages;   // a batch unit's first visual tile
         for (int j = 0; j < g.n1 + (g.batch ? 0 : g.n2); ++j, ++tc) {
           const int s = slot, buf = tc & 1;
-          if (!ptx::mbar_wait(k_full + s, kph, limit, p.status)) limit = kWaitNsAfterFault;
+          const uint32_t ph = kph;
           if (++slot == p.stages) {
             slot = 0;
             kph ^= 1u;
           }
+          if (buf != mid) continue;   // the other issuer's tile
+          if (!ptx::mbar_wait(k_full + s, ph, limit, p.status)) limit = kWaitNsAfterFault;
           if (tc >= 2 && !ptx::mbar_wait(a_empty + buf, (tc / 2 - 1) & 1, limit, p.status))
             limit = kWaitNsAfterFault;
           ptx::tc_fence_after();
@@ -327,7 +335,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!(g.batch && vi >= 0 && vi < g.n2)) ptx::mma_commit(k_empty + s);
           ptx::mma_commit(a_full + buf);  // the epilogue may read the buffer
         }
-        if (g.batch) {
+        if (g.batch && mid == 0) {
           // every sweep-1 accumulator read: the sweep-2 accumulators of all
           // visual tiles go side by side into TMEM columns j * n2c
           for (int k = 1; k <= 2; ++k) {
@@ -348,14 +356,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
         }
-        ptx::mma_commit(q_empty);   // every MMA of the unit is done with Q
+        ptx::mma_commit(q_empty);   // every MMA of this issuer in the unit is done with Q
         if (g.batch) {   // the next unit's accumulators wait for the batch to be read
           if (!ptx::mbar_wait(b_done, bu & 1, limit, p.status)) limit = kWaitNsAfterFault;
           ++bu;
         }
       }
     }
-  } else {
+  } else if (warp < 2 + kEpiWarps) {
     // ================= epilogue (16 warps)
     const int ew = warp - 2;
     const int q4 = warp & 3;                 // TMEM lane quarter: text rows 32*q4 ..
