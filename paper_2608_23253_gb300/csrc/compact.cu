@@ -39,13 +39,19 @@ __device__ __forceinline__ int out_image(const LayoutArgs& la, const int32_t* ke
 __device__ __forceinline__ void compact_rows(const LayoutArgs& la, const int32_t* keep_idx,
                                              const int32_t* keep_off, int n_tensors,
                                              const TensorSet& ts, int32_t* pos_ids,
-                                             long long total_rows, uint32_t* status, int visual) {
+                                             long long total_rows, uint32_t* status, int visual,
+                                             bool spread) {
   const int lane = threadIdx.x & 31;
   const long long warps = (long long)gridDim.x * (blockDim.x >> 5);
   // with no tensors the pass still writes the position ids
   const long long pairs = total_rows * (n_tensors > 0 ? n_tensors : 1);
-  for (long long pr = ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5; pr < pairs;
-       pr += warps) {
+  // spread: warp w of CTA c starts at pair w * gridDim.x + c, so consecutive
+  // pairs (an image's kept rows are consecutive) land on different SMs -- for
+  // kept rows already in L2, on the step's critical path; otherwise
+  // neighbouring rows stay in one CTA (DRAM locality)
+  const long long first = spread ? (long long)(threadIdx.x >> 5) * gridDim.x + blockIdx.x
+                                 : ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  for (long long pr = first; pr < pairs; pr += warps) {
     const int tix = (int)(pr / total_rows);
     const int r = (int)(pr - (long long)tix * total_rows);
     const int b = out_image(la, keep_off, r);
@@ -125,12 +131,13 @@ __global__ void __launch_bounds__(kCompactThreads)
   pdl_launch_dependents();
   if (early) {
     if (prefetch) prefetch_visual_rows(la, n_tensors, ts);
-    compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, 0);
+    compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, 0, false);
     pdl_wait();   // keep_idx comes from the previous kernel
-    compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, 1);
+    compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, 1,
+                 prefetch != 0);
   } else {
     pdl_wait();
-    compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, -1);
+    compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, -1, false);
   }
 }
 
