@@ -58,7 +58,7 @@ WORKLOADS = {
 KERNEL_SOURCES = ("score_unit.cu", "sm100_ptx.cuh", "device_common.cuh")
 NCU_TRAFFIC = {
     "cfg1": {"stage": "score", "kernel": "score_unit_kernel", "src": KERNEL_SOURCES,
-             "sha": "38ec279d0f5f240c", "bytes": 18230000},
+             "sha": "d9166a52ce292757", "bytes": 18224384},
 }
 
 
