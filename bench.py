@@ -58,7 +58,7 @@ WORKLOADS = {
 KERNEL_SOURCES = ("score_unit.cu", "sm100_ptx.cuh", "device_common.cuh")
 NCU_TRAFFIC = {
     "cfg1": {"stage": "score", "kernel": "score_unit_kernel", "src": KERNEL_SOURCES,
-             "sha": "d9166a52ce292757", "bytes": 18224384},
+             "sha": "0f6e171e130388e8", "bytes": 18230000},
 }
 
 

@@ -404,9 +404,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int c = et; c < ntp; c += kEpiThreads) wcol[c] = (c < NT) ? p.scale / (float)NT : 0.f;
         ptx::named_bar(1, kEpiThreads);
       }
-      // ---- pass C, plus the statistics of the unit's visual scores
-      float ls = 0.f, lm = kNegBig, av0 = 0.f, av1 = 0.f;
-      int na = 0;
+      // ---- pass C, plus the statistics of the unit's visual scores, kept
+      // online per lane (sum, max of a*log2e, sum of exp2 relative to it)
+      float st_s = 0.f, st_m = kNegBig, st_e = 0.f;
       for (int i = g.vf + ((grp - g.vf) & 3); i < g.vl; i += 4) {
         const int key = g.key_base + kTileKeys * i + row;
         float acc0 = 0.f, acc1 = 0.f;
@@ -426,30 +426,31 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (key >= g.S && key < g.S + g.NV) {
           const float a = acc0 + acc1;
           p.a_out[((size_t)g.l * la.H + g.h) * (size_t)la.sum_vis + g.v0 + (key - g.S)] = a;
-          ls += a;
-          lm = fmaxf(lm, a * kLog2e);
-          if (na == 0) av0 = a; else av1 = a;
-          ++na;
+          const float al = a * kLog2e, mnew = fmaxf(st_m, al);
+          st_e = st_e * fast_ex2(st_m - mnew) + fast_ex2(al - mnew);
+          st_m = mnew;
+          st_s += a;
         }
       }
-      ls = warp_reduce(ls, [](float x, float y) { return x + y; });
-      lm = warp_reduce(lm, [](float x, float y) { return fmaxf(x, y); });
-      if (lane == 0) red[ew] = make_float2(ls, lm);
-      ptx::named_bar(1, kEpiThreads);
-      float S = 0.f, M = kNegBig;
-      for (int w = 0; w < kEpiWarps; ++w) {
-        S += red[w].x;
-        M = fmaxf(M, red[w].y);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float s2 = __shfl_xor_sync(0xffffffffu, st_s, o);
+        const float m2 = __shfl_xor_sync(0xffffffffu, st_m, o);
+        const float e2 = __shfl_xor_sync(0xffffffffu, st_e, o);
+        st_s += s2;
+        lse_merge(st_m, st_e, m2, e2);
       }
-      float le = 0.f;
-      if (na > 0) le += fast_ex2(fmaf(av0, kLog2e, -M));
-      if (na > 1) le += fast_ex2(fmaf(av1, kLog2e, -M));
-      le = warp_reduce(le, [](float x, float y) { return x + y; });
-      if (lane == 0) red[kEpiWarps + ew] = make_float2(le, 0.f);
+      if (lane == 0) {
+        red[ew] = make_float2(st_s, st_m);
+        red[kEpiWarps + ew] = make_float2(st_e, 0.f);
+      }
       ptx::named_bar(1, kEpiThreads);
-      if (et == 0 && g.ok) {
-        float E = 0.f;
-        for (int w = 0; w < kEpiWarps; ++w) E += red[kEpiWarps + w].x;
+      if (et == 0 && g.ok) {   // the 16 warps in order
+        float S = 0.f, M = kNegBig, E = 0.f;
+        for (int w = 0; w < kEpiWarps; ++w) {
+          S += red[w].x;
+          lse_merge(M, E, red[w].y, red[kEpiWarps + w].x);
+        }
         p.stats[((size_t)g.b * la.L + g.l) * la.H + g.h] = stats_entry(S, M, E);
       }
       // TMEM of this unit fully read: the MMA warp may overwrite it
