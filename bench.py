@@ -37,17 +37,25 @@ import numpy as np  # noqa: E402
 
 METRIC = "pruning decisions/sec (images/s) at LLaVA-1.5 shape, K=64; % of HBM roofline"
 UNIT = "images/s"
-# name -> (config id, K, batch, description).  The default is the metric's
-# workload; the others exist for profiling and context lines.
+# name -> (config id, synth.config_spec keyword arguments, description).  The
+# default is the metric's workload; the others exist for profiling and context
+# lines.
 WORKLOADS = {
-    "cfg1": (1, 64, None, "llava-1.5-7b decision+compaction, batch 1, 35+576(24x24)+64 tokens, "
-                          "3 layers, 32x128 MHA, K=64"),
-    "cfg2": (2, 64, None, "llava-1.5-7b decision+compaction, batch 32, 35+576(24x24)+U[16,128] "
-                          "ragged text tokens, 3 layers, 32x128 MHA, K=64"),
-    "cfg3": (3, None, None, "qwen2-vl-7b decision+compaction, batch 16, grids 16x16..36x36, "
-                            "28q/4kv heads, 3 layers, K=11.1%"),
-    "cfg4": (4, None, None, "high-res decision+compaction, batch 8, 48x48/64x64 grids, 128 text, "
-                            "4 layers, 32x128 MHA, K=11%"),
+    "cfg1": (1, {"keep": 64}, "llava-1.5-7b decision+compaction, batch 1, 35+576(24x24)+64 "
+                              "tokens, 3 layers, 32x128 MHA, K=64"),
+    "cfg2": (2, {"keep": 64}, "llava-1.5-7b decision+compaction, batch 32, 35+576(24x24)+"
+                              "U[16,128] ragged text tokens, 3 layers, 32x128 MHA, K=64"),
+    "cfg3": (3, {}, "qwen2-vl-7b decision+compaction, batch 16, grids 16x16..36x36, "
+                    "28q/4kv heads, 3 layers, K=11.1%"),
+    "cfg4": (4, {}, "high-res decision+compaction, batch 8, 48x48/64x64 grids, 128 text, "
+                    "4 layers, 32x128 MHA, K=11%"),
+    # Sec. 4.5's two Qwen2-VL reduction ratios on dynamic-resolution grids
+    "qwen2vl-r66.7": (3, {"keep_ratio": 1 / 3, "dynamic_grids": True},
+                      "qwen2-vl-7b decision+compaction, batch 16, dynamic grids h,w in [12,48] "
+                      "(h*w <= 1296), 28q/4kv heads, 3 layers, K=N_V/3 (66.7% reduction)"),
+    "qwen2vl-r77.8": (3, {"keep_ratio": 2 / 9, "dynamic_grids": True},
+                      "qwen2-vl-7b decision+compaction, batch 16, dynamic grids h,w in [12,48] "
+                      "(h*w <= 1296), 28q/4kv heads, 3 layers, K=2N_V/9 (77.8% reduction)"),
 }
 
 # ncu dram__bytes_read.sum + dram__bytes_write.sum of one launch of the dominant
@@ -229,12 +237,12 @@ def cpu_oracle_rate(workload: str = "cfg1", seconds: float = 12.0, threads: int 
         "import sys,time,json;sys.path.insert(0,%r);import bench;"
         "from paper_2608_23253_gb300 import synth;"
         "from oracle import e2s_oracle as orc;"
-        "inp=synth.make_inputs(synth.config_spec(%d,keep=%r,batch=%r));p=orc.Params();"
+        "inp=synth.make_inputs(synth.config_spec(%d,**%r));p=orc.Params();"
         "bench.oracle_step(inp,p);n=0;t=time.perf_counter()\n"
         "while True:\n bench.oracle_step(inp,p);n+=1\n"
         " if time.perf_counter()-t>%f: break\n"
         "print(json.dumps({'images':n*inp.spec.B,'seconds':time.perf_counter()-t}))"
-    ) % (ROOT, WORKLOADS[workload][0], WORKLOADS[workload][1], WORKLOADS[workload][2], seconds)
+    ) % (ROOT, WORKLOADS[workload][0], WORKLOADS[workload][1], seconds)
     env = dict(os.environ)
     for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
         env[v] = str(threads)
@@ -263,7 +271,7 @@ def run_reference(args, world, rank):
         "impl": "reference", "metric": METRIC, "value": rate, "unit": UNIT, "n_gpus": args.gpus,
         "steps": info["images"], "warmup": 1, "ms_per_step": 1e3 / rate,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": WORKLOADS[args.workload][3]},
+        "data": "synthetic", "config": {"workload": WORKLOADS[args.workload][2]},
         "cpu_baseline": {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": f"decision+compaction of {info['images']} images of this "
                                    f"workload in {info['seconds']:.1f} s, 1 thread"},
@@ -283,8 +291,8 @@ def run_ours(args, world, rank, local):
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
-    cfg_id, keep, bsz, desc = WORKLOADS[args.workload]
-    inp = synth.make_inputs(synth.config_spec(cfg_id, keep=keep, batch=bsz), with_payload=True)
+    cfg_id, spec_kw, desc = WORKLOADS[args.workload]
+    inp = synth.make_inputs(synth.config_spec(cfg_id, **spec_kw), with_payload=True)
     s = inp.spec
     batch = Batch.from_inputs(inp, device=dev)
     dec = Decision(batch, inp.keep, e2s.params())
@@ -431,7 +439,8 @@ def run_ours(args, world, rank, local):
         "data": "synthetic",
         "config": {"workload": desc, "global_batch": batch.B * world, "seq_len": batch.sum_T,
                    "n_vis": int(inp.n_vis[0]), "n_text": int(inp.n_text[0]), "layers": L,
-                   "keep": int(inp.keep[0]), "score_mode": "causal_prob", "norm": "renorm",
+                   "keep": int(inp.keep[0]), "keep_total": int(inp.keep.sum()),
+                   "score_mode": "causal_prob", "norm": "renorm",
                    "parallelism": f"replicas{world}",
                    "l2": "flushed before every step (256 MiB write)"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

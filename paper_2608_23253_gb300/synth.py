@@ -92,7 +92,8 @@ def keep_for_ratio(n_vis: int, ratio: float) -> int:
 
 
 def config_spec(cfg: int, *, batch: Optional[int] = None, keep: Optional[int] = None,
-                images: Optional[int] = None) -> Spec:
+                images: Optional[int] = None, keep_ratio: Optional[float] = None,
+                dynamic_grids: bool = False) -> Spec:
     """Specs for the five workload configurations.
 
     cfg 0: tiny decision, B=1, L=2, MHA 32x128, 35 + 24x24 + 32, 20 random salient, K=64.
@@ -100,6 +101,10 @@ def config_spec(cfg: int, *, batch: Optional[int] = None, keep: Optional[int] = 
     cfg 2: cfg 1 per image, B=32, N_T ~ U[16,128] ragged, K in {64,128}.
     cfg 3: Qwen2-VL-7B, B=16, D=3584, 28 q / 4 kv heads, L=3, grids from
            {16x16, 24x32, 32x32, 36x36}, N_T=64, K = round(64/576 * N_V).
+           ``dynamic_grids`` draws any h, w in [12, 48] with h * w <= 1296 instead
+           (merged-patch grids of arbitrary image sizes, mostly not divisible by
+           G = 4); ``keep_ratio`` sets K = round(keep_ratio * N_V) (Sec. 4.5:
+           reductions of 66.7 % and 77.8 % keep 1/3 and 2/9).
     cfg 4: MHA 32x128, L=4, B=8 alternating 48x48 / 64x64 grids, N_T=128,
            salient blobs covering 5% of the grid, K = round(0.11 * N_V).
     ``batch``/``images`` shrink the batch for oracle-sized parity runs.
@@ -124,14 +129,22 @@ def config_spec(cfg: int, *, batch: Optional[int] = None, keep: Optional[int] = 
     if cfg == 3:
         b = 16 if batch is None else batch
         grids = [(16, 16), (24, 32), (32, 32), (36, 36)]
+        ratio = 64 / 576 if keep_ratio is None else keep_ratio
         ims = []
         for i in range(b):
             r = np.random.Generator(np.random.PCG64(1000 * 3 + i).jumped())
-            gh, gw = grids[int(r.integers(0, 4))]
+            if dynamic_grids:
+                while True:
+                    gh, gw = int(r.integers(12, 49)), int(r.integers(12, 49))
+                    if gh * gw <= 1296:
+                        break
+            else:
+                gh, gw = grids[int(r.integers(0, 4))]
             nv = gh * gw
             ims.append(ImageSpec(35, gh, gw, 64, round_half_even(40 * nv / 576), 3,
-                                 keep_for_ratio(nv, 64 / 576) if keep is None else keep))
-        return Spec("qwen2vl-gqa-ragged", 3, 3, 28, 4, 3584, ims)
+                                 keep_for_ratio(nv, ratio) if keep is None else keep))
+        name = "qwen2vl-gqa-dynres" if dynamic_grids else "qwen2vl-gqa-ragged"
+        return Spec(name, 3, 3, 28, 4, 3584, ims)
     if cfg == 4:
         b = 8 if batch is None else batch
         ims = []

@@ -99,15 +99,37 @@ def check_selection(gpu_keep, gpu_q_tilde, ref_q, n_vis, grid_h, grid_w, keep, l
         off += nv
 
 
-def oracle_keep_ok(ref, n_vis, keep, tol=TOL):
-    """Whether the oracle's own K-th / (K+1)-th margin exceeds tol for every image."""
-    off = 0
+def clear_margin_images(ref, n_vis, keep, tol=TOL):
+    """Images whose oracle K-th / (K+1)-th q~ margin exceeds tol."""
+    out, off = [], 0
     for b in range(len(n_vis)):
         nv = int(n_vis[b])
         kc = min(int(keep[b]), nv)
         if 0 < kc < nv:
             s = np.sort(ref["q_tilde"][off:off + nv])[::-1]
-            if s[kc - 1] - s[kc] <= tol:
-                return False
+            if s[kc - 1] - s[kc] > tol:
+                out.append(b)
+        else:
+            out.append(b)
         off += nv
-    return True
+    return out
+
+
+def oracle_keep_ok(ref, n_vis, keep, tol=TOL):
+    """Whether the oracle's own K-th / (K+1)-th margin exceeds tol for every image."""
+    return len(clear_margin_images(ref, n_vis, keep, tol)) == len(n_vis)
+
+
+def check_topk_of_own_scores(gpu_keep, gpu_q_tilde, n_vis, keep):
+    """The integer step taken in the kernel's precision: each image's retained
+    set is the Top-K of the q~ the GPU wrote (float32, ties to the lower
+    index), in ascending order."""
+    off = 0
+    for b in range(len(n_vis)):
+        nv = int(n_vis[b])
+        kc = min(int(keep[b]), nv)
+        qt = np.asarray(gpu_q_tilde[off:off + nv], dtype=np.float32)
+        order = np.lexsort((np.arange(nv), -qt.astype(np.float64)))
+        want = np.sort(order[:kc])
+        assert np.array_equal(np.asarray(gpu_keep[b])[:kc], want), f"image {b}: not Top-K of q~"
+        off += nv

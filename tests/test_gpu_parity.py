@@ -4,13 +4,16 @@ All five configurations run at their full per-image shapes; configuration 4
 (high-resolution, 2304 and 4096 visual tokens) is cut to two images here and
 run at its full batch of eight in test_gpu_fullsize.py.
 """
+import functools
+
 import numpy as np
 import pytest
 import torch
 
 from oracle import e2s_oracle as orc
 from tests import parity
-from tests.gpu_helpers import config_inputs, config_oracle, device, run_gpu
+from paper_2608_23253_gb300 import synth
+from tests.gpu_helpers import config_inputs, config_oracle, device, run_gpu, run_oracle
 
 pytestmark = pytest.mark.gpu
 
@@ -42,6 +45,7 @@ def test_decision_parity(case, path, mode):
     parity.check_floats(gpu, ref)
     parity.check_selection(gpu["keep"], gpu["q_tilde"], ref["q"], inp.n_vis, inp.grid_h,
                            inp.grid_w, inp.keep, 0.1, 4)
+    parity.check_topk_of_own_scores(gpu["keep"], gpu["q_tilde"], inp.n_vis, inp.keep)
     if parity.oracle_keep_ok(ref, inp.n_vis, inp.keep):
         for b in range(inp.spec.B):
             assert np.array_equal(gpu["keep"][b], ref["keep"][b])
@@ -107,11 +111,14 @@ def test_prune_whole_step(cfg, batch):
     """e2s_prune (decide, then compaction whose fixed rows overlap the decision):
     the decision matches the oracle, and every output row is the oracle's
     compaction of the keep set the GPU chose, bit for bit."""
+    inp = config_inputs(cfg, batch, None, True)
+    _check_prune(inp, config_oracle(cfg, batch, None, "causal"))
+
+
+def _check_prune(inp, ref):
     from paper_2608_23253_gb300 import e2s
     from paper_2608_23253_gb300.decision import Batch, Decision, bf16_tensor
     dev = device()
-    inp = config_inputs(cfg, batch, None, True)
-    ref = config_oracle(cfg, batch, None, "causal")
     dec = Decision(Batch.from_inputs(inp, device=dev), inp.keep, e2s.params())
     L = inp.spec.L
     host = [inp.hidden] + [inp.k[l].reshape(inp.k.shape[1], -1) for l in range(L)] + \
@@ -129,6 +136,7 @@ def test_prune_whole_step(cfg, batch):
     parity.check_floats(gpu, ref)
     parity.check_selection(gpu["keep"], gpu["q_tilde"], ref["q"], inp.n_vis, inp.grid_h,
                            inp.grid_w, inp.keep, 0.1, 4)
+    parity.check_topk_of_own_scores(gpu["keep"], gpu["q_tilde"], inp.n_vis, inp.keep)
     if parity.oracle_keep_ok(ref, inp.n_vis, inp.keep):
         for b in range(inp.spec.B):
             assert np.array_equal(gpu["keep"][b], ref["keep"][b])
@@ -137,3 +145,34 @@ def test_prune_whole_step(cfg, batch):
         assert np.array_equal(d_.cpu().view(torch.int16).numpy().view(np.uint16), want)
     assert np.array_equal(pos.cpu().numpy(),
                           orc.position_ids(inp.n_sys, inp.n_vis, inp.n_text, gpu["keep"]))
+
+
+# Sec. 4.5 evaluates Qwen2-VL-7B at visual-token reductions of 66.7 % and
+# 77.8 % (K = N_V / 3 and 2 N_V / 9 per image).  Its dynamic resolution gives
+# merged-patch grids of any shape, most of them not divisible by G = 4.
+DYNRES = {"r66.7": 1 / 3, "r77.8": 2 / 9}
+
+
+@functools.lru_cache(maxsize=None)
+def _dynres(ratio: str):
+    inp = synth.make_inputs(synth.config_spec(3, keep_ratio=DYNRES[ratio], dynamic_grids=True),
+                            with_payload=True)
+    return inp, run_oracle(inp, "causal")
+
+
+@pytest.mark.parametrize("path", ["prune", "fuse_select", "separate"])
+@pytest.mark.parametrize("ratio", sorted(DYNRES))
+def test_qwen2vl_dynamic_resolution(ratio, path):
+    inp, ref = _dynres(ratio)
+    assert sum(int(h) % 4 != 0 or int(w) % 4 != 0 for h, w in zip(inp.grid_h, inp.grid_w)) >= 8
+    if path == "prune":
+        _check_prune(inp, ref)
+        return
+    gpu = run_gpu(inp, "causal", path=path)
+    assert gpu["status"] == 0, gpu["status"]
+    parity.check_floats(gpu, ref)
+    parity.check_selection(gpu["keep"], gpu["q_tilde"], ref["q"], inp.n_vis, inp.grid_h,
+                           inp.grid_w, inp.keep, 0.1, 4)
+    parity.check_topk_of_own_scores(gpu["keep"], gpu["q_tilde"], inp.n_vis, inp.keep)
+    for b in parity.clear_margin_images(ref, inp.n_vis, inp.keep):
+        assert np.array_equal(gpu["keep"][b], ref["keep"][b])
