@@ -27,18 +27,29 @@
 namespace e2s {
 namespace {
 
-constexpr int kTok = 64;                           // visual tokens per CTA
-constexpr int kRow = kTok;                         // staged row stride (floats)
 constexpr int kDecThreads = 256;
-constexpr int kLayerLanes = kDecThreads / kTok;    // layers handled side by side
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr size_t kDecSmemBudget = 160u << 10;
 
+// Visual tokens per CTA.  64 when the batch fills the GPU; 16 for small
+// batches, where the CTA's 256 threads split each (token, layer)'s heads four
+// ways so the per-thread walk over the heads is four times shorter.
+template <int TOK>
+struct DecTile {
+  static constexpr int kTok = TOK;
+  // staged row stride (floats): with heads split four ways (head h = 4i + g on
+  // lane group g), 24 keeps the four groups of a warp in distinct banks
+  static constexpr int kRow = TOK == 64 ? 64 : 24;
+  static constexpr int kHeadSplit = TOK == 64 ? 1 : 4;
+  static constexpr int kLayerLanes = kDecThreads / (TOK * kHeadSplit);   // layers side by side
+};
+
 // [L][H] statistics, [L][kTok] layer masses and head sums, then the staged
 // scores [L][H][kRow] (reused as the select's keys and cell ids).
+template <int TOK>
 __host__ __device__ inline size_t dec_smem_bytes(int L, int H, int max_vis) {
-  const size_t st = (size_t)L * H * 16 + (size_t)L * kTok * 20;
-  const size_t a = (size_t)L * H * kRow * 4;
+  const size_t st = (size_t)L * H * 16 + (size_t)L * TOK * 20;
+  const size_t a = (size_t)L * H * DecTile<TOK>::kRow * 4;
   const size_t sel = (size_t)max_vis * 5;
   return st + (a > sel ? a : sel);
 }
@@ -79,7 +90,10 @@ __device__ __forceinline__ float support_p(float a, float4 st, int softmax, floa
   return x * fast_rcp(1.f + x);                     // Eq. 9
 }
 
+template <int TOK>
 __global__ void __launch_bounds__(kDecThreads) decide_kernel(const DecArgs p) {
+  constexpr int kTok = DecTile<TOK>::kTok, kRow = DecTile<TOK>::kRow;
+  constexpr int kSplit = DecTile<TOK>::kHeadSplit, kLayerLanes = DecTile<TOK>::kLayerLanes;
   extern __shared__ __align__(16) uint8_t dec_smem[];
   __shared__ SelectSmem ss;
   __shared__ int is_last;
@@ -127,7 +141,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const DecArgs p) {
     }
   } else {
     for (int idx = tid; idx < L * H * kTok; idx += kDecThreads) {
-      const int jj = idx & (kTok - 1), lh = idx >> 6;
+      const int jj = idx & (kTok - 1), lh = idx / kTok;
       if (jj < ntok) ptx::cp_async4(A + lh * kRow + jj, p.a + (size_t)lh * plane + v0 + n0 + jj);
     }
   }
@@ -138,7 +152,7 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const DecArgs p) {
   const float N = (float)NV;
   const float invN = NV > 0 ? 1.f / N : 0.f;
   const float inv_h = 1.f / (float)H;
-  {
+  if constexpr (kSplit == 1) {
     const int j = tid & (kTok - 1);
     for (int l = tid / kTok; l < L; l += kLayerLanes) {
       if (j >= ntok) continue;
@@ -167,6 +181,49 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const DecArgs p) {
       M_s[l * kTok + j] = m4;
       SA_s[l * kTok + j] = sum_a;
       if (p.mass_out) p.mass_out[(size_t)l * plane + v0 + n0 + j] = m4;
+    }
+  } else {
+    // lane = (token & 7) + 8 g: the four lanes of a (token, layer) take heads
+    // h = g, g + 4, ... and combine their partial sums with two shuffles;
+    // warp w takes tokens 8 (w & 1) .. + 7 of layer lane w >> 1
+    const int lane = tid & 31, wp = tid >> 5, g = lane >> 3;
+    const int j = (lane & 7) + 8 * (wp & 1);
+    for (int l = wp >> 1; l < L; l += kLayerLanes) {
+      float* Ac = A + (size_t)l * H * kRow + j;
+      const float4* sl = st_s + (size_t)l * H;
+      float sum_p = 0.f, sum_a = 0.f;
+#pragma unroll 4
+      for (int h = g; h < H; h += kSplit) {
+        const float av = Ac[h * kRow];
+        const float pv = support_p(av, sl[h], p.softmax, N, invN);
+        sum_a += av;
+        sum_p += pv;
+        Ac[h * kRow] = pv;
+      }
+      sum_p += __shfl_xor_sync(0xffffffffu, sum_p, 8);
+      sum_p += __shfl_xor_sync(0xffffffffu, sum_p, 16);
+      sum_a += __shfl_xor_sync(0xffffffffu, sum_a, 8);
+      sum_a += __shfl_xor_sync(0xffffffffu, sum_a, 16);
+      const float p_bar = sum_p * inv_h;
+      float clar = 0.f, dev = 0.f;
+#pragma unroll 4
+      for (int h = g; h < H; h += kSplit) {
+        const float pv = Ac[h * kRow];
+        clar += pv - 0.5f;
+        dev += fabsf(pv - p_bar);
+      }
+      clar += __shfl_xor_sync(0xffffffffu, clar, 8);
+      clar += __shfl_xor_sync(0xffffffffu, clar, 16);
+      dev += __shfl_xor_sync(0xffffffffu, dev, 8);
+      dev += __shfl_xor_sync(0xffffffffu, dev, 16);
+      float rho = (2.f * inv_h) * fabsf(clar) * (1.f - (2.f * inv_h) * dev);  // Eq. 10
+      if (p.flags & E2S_NO_RELIABILITY) rho = 1.f;
+      const float4 m4 = make_float4(rho * p_bar, rho * (1.f - p_bar), 1.f - rho, p_bar);  // Eq. 11
+      if (g == 0 && j < ntok) {
+        M_s[l * kTok + j] = m4;
+        SA_s[l * kTok + j] = sum_a;
+        if (p.mass_out) p.mass_out[(size_t)l * plane + v0 + n0 + j] = m4;
+      }
     }
   }
   __syncthreads();
@@ -249,7 +306,8 @@ __global__ void __launch_bounds__(kDecThreads) decide_kernel(const DecArgs p) {
 }  // namespace
 
 bool decide_fits(const LayoutArgs& la) {
-  return dec_smem_bytes(la.L, la.H, la.max_vis) <= kDecSmemBudget;
+  return dec_smem_bytes<64>(la.L, la.H, la.max_vis) <= kDecSmemBudget &&
+         dec_smem_bytes<16>(la.L, la.H, la.max_vis) <= kDecSmemBudget;
 }
 
 cudaError_t launch_decide(const LayoutArgs& la, int norm_softmax, uint32_t flags, float lambda,
@@ -270,7 +328,10 @@ cudaError_t launch_decide(const LayoutArgs& la, int norm_softmax, uint32_t flags
   p.flags = flags;
   p.lam = lambda;
   p.G = G;
-  p.blocks_per_image = (la.max_vis + kTok - 1) / kTok;
+  // 16-token CTAs while the 64-token grid would leave most SMs idle
+  const bool small = (int64_t)la.B * ((la.max_vis + 63) / 64) < (int64_t)sm_count();
+  const int tok = small ? 16 : 64;
+  p.blocks_per_image = (la.max_vis + tok - 1) / tok;
   p.a = a;
   p.stats = stats;
   p.prior = reinterpret_cast<const float4*>(prior);
@@ -286,9 +347,12 @@ cudaError_t launch_decide(const LayoutArgs& la, int norm_softmax, uint32_t flags
   p.cell_best = reinterpret_cast<unsigned long long*>(scratch);
   p.counters = scratch + (size_t)2 * kDecideCells * la.B;
   p.status = status;
-  const size_t smem = dec_smem_bytes(la.L, la.H, la.max_vis);
-  return launch_kernel(decide_kernel, dim3((unsigned)(la.B * p.blocks_per_image)),
-                       dim3(kDecThreads), smem, st, 0, true, p);
+  const dim3 grid((unsigned)(la.B * p.blocks_per_image));
+  if (small)
+    return launch_kernel(decide_kernel<16>, grid, dim3(kDecThreads),
+                         dec_smem_bytes<16>(la.L, la.H, la.max_vis), st, 0, true, p);
+  return launch_kernel(decide_kernel<64>, grid, dim3(kDecThreads),
+                       dec_smem_bytes<64>(la.L, la.H, la.max_vis), st, 0, true, p);
 }
 
 }  // namespace e2s
