@@ -124,6 +124,26 @@ e2s_status e2s_score(const e2s_layout* layout, const e2s_params* params,
                      const void* k, int64_t k_row_stride,
                      float* a_out, void* ws, size_t ws_bytes, void* stream);
 
+/* Text-to-visual score reusing the pruning layer's own attention pass (Sec. 6
+ * names lower-overhead evidence caching as future work; taking the attention
+ * pass's row normalisers is this library's reading of it).  A flash-attention forward of the layer already
+ * returns, for every query row, the natural-log log-sum-exp of its scaled
+ * logits Q_t K_j / sqrt(d) over the row's causal prefix (j = 0 .. S+N_V+t).
+ * Given those of the text rows, the CAUSAL_PROB score needs only the visual
+ * key tiles, in one pass: a[l][h][n] = mean over t of
+ * exp(Q_t K_n / sqrt(d) - lse_t), with no sweep over the whole prefix for the
+ * row normalisers.
+ *   lse_text  fp32 [L][H][sum_text], device, 4-byte aligned:
+ *             lse_text[(l*H + h)*sum_text + text_off[b] + t] for text row t of
+ *             image b, query head h, layer l.  Its accuracy bounds that of a.
+ * Other arguments, the results and the Eq. 8 statistics left in the workspace
+ * are those of e2s_score.  E2S_ERR_UNSUPPORTED unless score_mode is
+ * CAUSAL_PROB, E2S_SIMT_SCORE is clear and max_text <= 128. */
+e2s_status e2s_score_lse(const e2s_layout* layout, const e2s_params* params,
+                         const void* q_text, int64_t q_row_stride,
+                         const void* k, int64_t k_row_stride, const float* lse_text,
+                         float* a_out, void* ws, size_t ws_bytes, void* stream);
+
 /* The whole pruning decision of one step in two launches: e2s_score, then
  * evidence, fusion and selection (Sec. 3.1 and 4.1-4.3, Eqs. 1 and 8-23).
  * Arguments have the meaning they have in e2s_score, e2s_fuse and e2s_select;
@@ -145,6 +165,17 @@ e2s_status e2s_decide(const e2s_layout* layout, const e2s_params* params,
                       const int32_t* keep_count, const int32_t* keep_off, int32_t sum_keep,
                       int32_t* keep_idx, float* q_tilde_out,
                       void* ws, size_t ws_bytes, void* stream);
+
+/* e2s_decide with its score taken as e2s_score_lse takes it (same lse_text
+ * argument and restrictions). */
+e2s_status e2s_decide_lse(const e2s_layout* layout, const e2s_params* params,
+                          const void* q_text, int64_t q_row_stride,
+                          const void* k, int64_t k_row_stride, const float* lse_text,
+                          const int32_t* cand, const float* prior, float* a_out,
+                          float* mass_out, float* fused_out, float* q_out,
+                          const int32_t* keep_count, const int32_t* keep_off, int32_t sum_keep,
+                          int32_t* keep_idx, float* q_tilde_out,
+                          void* ws, size_t ws_bytes, void* stream);
 
 /* One complete pruning step: e2s_decide followed by e2s_compact, three
  * launches (Algorithm 1, one pruning layer; Sec. 3.1 and 4.1-4.3).  Arguments

@@ -85,6 +85,22 @@ def causal_attention_rows(Q: np.ndarray, K_all: np.ndarray, first_text_pos: int)
     return e / e.sum(axis=1, keepdims=True)
 
 
+def causal_row_lse(Q: np.ndarray, K_all: np.ndarray, first_text_pos: int) -> np.ndarray:
+    """Natural-log normaliser of each text row's causal softmax (Sec. 3.1):
+    lse_t = log sum_{j <= first_text_pos + t} exp(Q_t K_j / sqrt(d)), so that
+    P_{t,j} = exp(Q_t K_j / sqrt(d) - lse_t).  A flash-attention forward of the
+    layer returns this value for every query row; the score can start from it.
+    """
+    d = Q.shape[1]
+    T = K_all.shape[0]
+    logits = Q @ K_all.T / np.sqrt(d)          # [N_T, T]
+    pos = first_text_pos + np.arange(Q.shape[0])
+    visible = np.arange(T)[None, :] <= pos[:, None]
+    z = np.where(visible, logits, -np.inf)
+    m = z.max(axis=1)
+    return m + np.log(np.exp(z - m[:, None]).sum(axis=1))
+
+
 def score_causal_prob(Q: np.ndarray, K_all: np.ndarray, S: int, N_V: int) -> np.ndarray:
     """a_n = (1/N_T) sum_t P_{t, S+n}: mean text-to-visual attention probability."""
     P = causal_attention_rows(Q, K_all, S + N_V)
@@ -272,6 +288,26 @@ def image_scores(q_text, k, b, lay, H_kv, score_mode) -> np.ndarray:
             else:
                 a[l, h] = score_causal_prob(Q, widen_bf16(k[l, t0:t0 + T, h // group]), S, N_V)
     return a
+
+
+def text_row_lse(q_text, k, n_sys, n_vis, n_text, *, H_kv: int) -> np.ndarray:
+    """lse [L, H, sum N_T] of every text row of a packed batch (causal_row_lse
+    per image, layer and query head), laid out as the rows of q_text."""
+    L, sum_text, H, d = q_text.shape
+    group = H // H_kv
+    out = np.zeros((L, H, sum_text))
+    t0 = x0 = 0
+    for b in range(len(n_sys)):
+        S, N_V, N_T = int(n_sys[b]), int(n_vis[b]), int(n_text[b])
+        T = S + N_V + N_T
+        for l in range(L):
+            for h in range(H):
+                Q = widen_bf16(q_text[l, x0:x0 + N_T, h])
+                out[l, h, x0:x0 + N_T] = causal_row_lse(
+                    Q, widen_bf16(k[l, t0:t0 + T, h // group]), S + N_V)
+        t0 += T
+        x0 += N_T
+    return out
 
 
 def image_evidence(a: np.ndarray, params: Params) -> Dict[str, np.ndarray]:

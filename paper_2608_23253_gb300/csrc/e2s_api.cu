@@ -87,11 +87,17 @@ e2s_status check_score_args(const e2s_layout* layout, const void* q_text, int64_
 }
 
 // Score launch shared by e2s_score and e2s_decide; the decision scratch it
-// zeroes may be null.
+// zeroes may be null.  With lse_text (the *_lse entry points) only the
+// streaming kernel's single visual pass runs.
 e2s_status run_score(const e2s_layout* layout, const e2s_params* params, const void* q_text,
                      int64_t q_row_stride, const void* k, int64_t k_row_stride, float* a_out,
-                     void* ws, uint32_t* counters, cudaStream_t st) {
+                     void* ws, uint32_t* counters, cudaStream_t st,
+                     const float* lse_text = nullptr) {
   const LayoutArgs la = layout_args(layout);
+  if (lse_text)
+    return from_cuda(launch_score_stream(la, params->score_mode, q_text, q_row_stride, k,
+                                         k_row_stride, a_out, stats_ptr(ws), counters,
+                                         status_word(ws), st, lse_text));
   if (params->flags & E2S_SIMT_SCORE)
     return from_cuda(launch_score_simt(la, params->score_mode, q_text, q_row_stride, k,
                                        k_row_stride, a_out, stats_ptr(ws), counters,
@@ -128,10 +134,11 @@ e2s_status run_decide(const e2s_layout* layout, const e2s_params* params, const 
                       const int32_t* cand, const float* prior, float* a_out, float* mass_out,
                       float* fused_out, float* q_out, const int32_t* keep_count,
                       const int32_t* keep_off, int32_t sum_keep, int32_t* keep_idx,
-                      float* q_tilde_out, void* ws, cudaStream_t st) {
+                      float* q_tilde_out, void* ws, cudaStream_t st,
+                      const float* lse_text = nullptr) {
   uint32_t* scratch = decide_scratch_ptr(ws, layout);
   E2S_TRY(run_score(layout, params, q_text, q_row_stride, k, k_row_stride, a_out, ws, scratch,
-                    st));
+                    st, lse_text));
   int unsupported = 0;
   const cudaError_t e =
       launch_decide(layout_args(layout), norm_is_softmax(params), params->flags, params->lambda,
@@ -140,6 +147,17 @@ e2s_status run_decide(const e2s_layout* layout, const e2s_params* params, const 
                     status_word(ws), st, &unsupported);
   if (unsupported) return E2S_ERR_UNSUPPORTED;
   return from_cuda(e);
+}
+
+// The text rows' lse given: causal-probability scores on the streaming kernel.
+e2s_status check_lse_args(const e2s_layout* layout, const e2s_params* params,
+                          const float* lse_text) {
+  if (!lse_text) return E2S_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(lse_text) & 3u) != 0) return E2S_ERR_ALIGNMENT;
+  if (params->score_mode != E2S_SCORE_CAUSAL_PROB || (params->flags & E2S_SIMT_SCORE))
+    return E2S_ERR_UNSUPPORTED;
+  if (!score_stream_fits(layout_args(layout))) return E2S_ERR_UNSUPPORTED;
+  return E2S_OK;
 }
 
 e2s_status check_compact_args(const e2s_layout* layout, const int32_t* keep_idx,
@@ -180,6 +198,35 @@ e2s_status e2s_score(const e2s_layout* layout, const e2s_params* params, const v
   E2S_TRY(check_score_args(layout, q_text, q_row_stride, k, k_row_stride, a_out));
   return run_score(layout, params, q_text, q_row_stride, k, k_row_stride, a_out, ws, nullptr,
                    static_cast<cudaStream_t>(stream));
+}
+
+e2s_status e2s_score_lse(const e2s_layout* layout, const e2s_params* params, const void* q_text,
+                         int64_t q_row_stride, const void* k, int64_t k_row_stride,
+                         const float* lse_text, float* a_out, void* ws, size_t ws_bytes,
+                         void* stream) {
+  E2S_TRY(check_layout(layout));
+  E2S_TRY(check_params(params));
+  E2S_TRY(check_ws(layout, ws, ws_bytes));
+  E2S_TRY(check_score_args(layout, q_text, q_row_stride, k, k_row_stride, a_out));
+  E2S_TRY(check_lse_args(layout, params, lse_text));
+  return run_score(layout, params, q_text, q_row_stride, k, k_row_stride, a_out, ws, nullptr,
+                   static_cast<cudaStream_t>(stream), lse_text);
+}
+
+e2s_status e2s_decide_lse(const e2s_layout* layout, const e2s_params* params,
+                          const void* q_text, int64_t q_row_stride, const void* k,
+                          int64_t k_row_stride, const float* lse_text, const int32_t* cand,
+                          const float* prior, float* a_out, float* mass_out, float* fused_out,
+                          float* q_out, const int32_t* keep_count, const int32_t* keep_off,
+                          int32_t sum_keep, int32_t* keep_idx, float* q_tilde_out, void* ws,
+                          size_t ws_bytes, void* stream) {
+  E2S_TRY(check_decide_args(layout, params, q_text, q_row_stride, k, k_row_stride, prior, a_out,
+                            mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
+                            ws, ws_bytes));
+  E2S_TRY(check_lse_args(layout, params, lse_text));
+  return run_decide(layout, params, q_text, q_row_stride, k, k_row_stride, cand, prior, a_out,
+                    mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
+                    q_tilde_out, ws, static_cast<cudaStream_t>(stream), lse_text);
 }
 
 e2s_status e2s_decide(const e2s_layout* layout, const e2s_params* params, const void* q_text,

@@ -69,11 +69,14 @@ cudaError_t launch_score_tc(const LayoutArgs& la, int mode, const void* q, int64
                             const void* k, int64_t k_stride, float* a_out, float4* stats,
                             uint32_t* counters, uint32_t* status, cudaStream_t st,
                             int* unsupported);
-// Streaming score kernel (long sequences, GQA; at most 128 text rows).
+// Streaming score kernel (long sequences, GQA; at most 128 text rows).  With
+// lse_in (natural-log lse of every text row, [L][H][sum_text]) it skips the
+// normaliser sweep and streams only the visual key tiles.
 bool score_stream_fits(const LayoutArgs& la);
 cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                                 const void* k, int64_t k_stride, float* a_out, float4* stats,
-                                uint32_t* counters, uint32_t* status, cudaStream_t st);
+                                uint32_t* counters, uint32_t* status, cudaStream_t st,
+                                const float* lse_in = nullptr);
 // Persistent single-CTA-per-unit score kernel and its applicability tests.
 bool score_unit_fits(const LayoutArgs& la, int mode);
 bool score_unit_single_group(const LayoutArgs& la, int mode);

@@ -68,6 +68,7 @@ struct StreamArgs {
   int num_units;
   float scale;          // 1 / sqrt(d)
   float scale_log2;     // log2(e) / sqrt(d)
+  const float* lse_in;  // nullable: natural-log lse of every text row, [L][H][sum_text]
   float* a_out;
   float4* stats;        // per (image, layer, head) statistics of the visual scores
   uint32_t* counters;   // nullable: decision scratch to zero
@@ -146,10 +147,12 @@ __device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit) {
   g.n2 = g.ok ? (g.NV + kTileKeys - 1) / kTileKeys : 0;
   g.n_st = (g.S + kTileKeys - 1) / kTileKeys;
   g.n_tt = max(0, (g.NV + g.NT + kTileKeys - 1) / kTileKeys - g.n2);
-  g.batch = HPU == 1 && g.ok && causal && g.n2 >= 1 && g.n2 <= kMaxBatch &&
+  // with the rows' lse given (from the layer's attention pass) there is no sweep 1
+  const bool given = p.lse_in != nullptr;
+  g.batch = !given && HPU == 1 && g.ok && causal && g.n2 >= 1 && g.n2 <= kMaxBatch &&
             g.n2 * sweep2_cols<HPU>(g.NT) <= kTmemCols && g.n2 + g.n_tt <= p.stages;
   g.kfirst = g.batch ? g.S - kTileKeys * g.n_st : 0;
-  g.n1 = !(g.ok && causal) ? 0
+  g.n1 = !(g.ok && causal) || given ? 0
          : g.batch ? g.n_st + g.n2 + g.n_tt : (T + kTileKeys - 1) / kTileKeys;
   return g;
 }
@@ -432,8 +435,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) ptx::mbar_arrive(a_empty + buf);
       }
       // ---- merge the four column groups: lse per row (log2 domain), published
-      // per text row for sweep 2
-      if (causal) {
+      // per text row for sweep 2 (or taken from the caller's attention pass)
+      if (causal && p.lse_in != nullptr) {
+        if (cg == 0 && (!SPLIT || lrow < kRows / 2))
+          lse_s[lrow] = tvalid ? __ldg(p.lse_in + ((size_t)g.l * la.H + g.h + hs) * la.sum_text +
+                                       g.x0 + t) * kLog2e
+                               : kNegBig;
+        ptx::named_bar(1, kEpiThreads);
+      } else if (causal) {
         ms[cg * kRows + lrow] = make_float2(m, ssum);
         ptx::named_bar(1, kEpiThreads);
         // partials of this row: four column groups (and, SPLIT, both lane halves)
@@ -638,8 +647,10 @@ bool score_stream_fits(const LayoutArgs& la) {
 
 cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                                 const void* k, int64_t k_stride, float* a_out, float4* stats,
-                                uint32_t* counters, uint32_t* status, cudaStream_t st) {
+                                uint32_t* counters, uint32_t* status, cudaStream_t st,
+                                const float* lse_in) {
   StreamArgs p;
+  p.lse_in = lse_in;
   p.la = la;
   p.mode = mode;
   p.group = la.H / la.H_kv;

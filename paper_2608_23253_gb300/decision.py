@@ -98,10 +98,16 @@ class Decision:
 
     # -- the four ABI calls
     def score(self, q_text: torch.Tensor, k: torch.Tensor, stream=None,
-              q_row_stride: Optional[int] = None, k_row_stride: Optional[int] = None) -> None:
+              q_row_stride: Optional[int] = None, k_row_stride: Optional[int] = None,
+              lse: Optional[torch.Tensor] = None) -> None:
+        """e2s_score, or e2s_score_lse when the text rows' attention lse is given."""
         b = self.batch
         qs = q_row_stride if q_row_stride is not None else b.H * b.d
         ks = k_row_stride if k_row_stride is not None else b.H_kv * b.d
+        if lse is not None:
+            e2s.check(e2s.e2s_score_lse(b.layout, self.params, q_text, qs, k, ks, lse, self.a,
+                                        self.ws, self.ws_bytes, stream), "e2s_score_lse")
+            return
         e2s.check(e2s.e2s_score(b.layout, self.params, q_text, qs, k, ks, self.a, self.ws,
                                 self.ws_bytes, stream), "e2s_score")
 
@@ -135,11 +141,20 @@ class Decision:
 
     def decide(self, q_text: torch.Tensor, k: torch.Tensor, prior: Optional[torch.Tensor] = None,
                cand: Optional[torch.Tensor] = None, stream=None,
-               q_row_stride: Optional[int] = None, k_row_stride: Optional[int] = None) -> None:
-        """score + fuse + select in two launches (e2s_decide)."""
+               q_row_stride: Optional[int] = None, k_row_stride: Optional[int] = None,
+               lse: Optional[torch.Tensor] = None) -> None:
+        """score + fuse + select in two launches (e2s_decide; e2s_decide_lse when
+        the text rows' attention lse is given)."""
         b = self.batch
         qs = q_row_stride if q_row_stride is not None else b.H * b.d
         ks = k_row_stride if k_row_stride is not None else b.H_kv * b.d
+        if lse is not None:
+            e2s.check(e2s.e2s_decide_lse(b.layout, self.params, q_text, qs, k, ks, lse, cand,
+                                         prior, self.a, self.mass, self.fused, self.q,
+                                         self.keep_count, self.keep_off, self.sum_keep,
+                                         self.keep_idx, self.q_tilde, self.ws, self.ws_bytes,
+                                         stream), "e2s_decide_lse")
+            return
         e2s.check(e2s.e2s_decide(b.layout, self.params, q_text, qs, k, ks, cand, prior, self.a,
                                  self.mass, self.fused, self.q, self.keep_count, self.keep_off,
                                  self.sum_keep, self.keep_idx, self.q_tilde, self.ws,

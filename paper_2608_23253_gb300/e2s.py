@@ -73,8 +73,11 @@ _sz = ctypes.c_size_t
 _SIGS = {
     "e2s_workspace_size": (_sz, [_LP, _PP]),
     "e2s_score": (ctypes.c_int, [_LP, _PP, _vp, _i64, _vp, _i64, _vp, _vp, _sz, _vp]),
+    "e2s_score_lse": (ctypes.c_int, [_LP, _PP, _vp, _i64, _vp, _i64, _vp, _vp, _vp, _sz, _vp]),
     "e2s_decide": (ctypes.c_int, [_LP, _PP, _vp, _i64, _vp, _i64, _vp, _vp, _vp, _vp, _vp, _vp,
                                    _vp, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
+    "e2s_decide_lse": (ctypes.c_int, [_LP, _PP, _vp, _i64, _vp, _i64, _vp, _vp, _vp, _vp, _vp,
+                                       _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _sz, _vp]),
     "e2s_prune": (ctypes.c_int, [_LP, _PP, _vp, _i64, _vp, _i64, _vp, _vp, _vp, _vp, _vp, _vp,
                                   _vp, _vp, _i32, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _sz,
                                   _vp]),
@@ -131,6 +134,23 @@ def e2s_score(layout, params_, q_text, q_row_stride, k, k_row_stride, a_out, ws,
               stream=None) -> int:
     return lib.e2s_score(_ref(layout), _ref(params_), _ptr(q_text), q_row_stride, _ptr(k),
                          k_row_stride, _ptr(a_out), _ptr(ws), ws_bytes, _stream(stream))
+
+
+def e2s_score_lse(layout, params_, q_text, q_row_stride, k, k_row_stride, lse_text, a_out, ws,
+                  ws_bytes, stream=None) -> int:
+    return lib.e2s_score_lse(_ref(layout), _ref(params_), _ptr(q_text), q_row_stride, _ptr(k),
+                             k_row_stride, _ptr(lse_text), _ptr(a_out), _ptr(ws), ws_bytes,
+                             _stream(stream))
+
+
+def e2s_decide_lse(layout, params_, q_text, q_row_stride, k, k_row_stride, lse_text, cand, prior,
+                   a_out, mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
+                   q_tilde_out, ws, ws_bytes, stream=None) -> int:
+    return lib.e2s_decide_lse(_ref(layout), _ref(params_), _ptr(q_text), q_row_stride, _ptr(k),
+                              k_row_stride, _ptr(lse_text), _ptr(cand), _ptr(prior), _ptr(a_out),
+                              _ptr(mass_out), _ptr(fused_out), _ptr(q_out), _ptr(keep_count),
+                              _ptr(keep_off), sum_keep, _ptr(keep_idx), _ptr(q_tilde_out),
+                              _ptr(ws), ws_bytes, _stream(stream))
 
 
 def e2s_decide(layout, params_, q_text, q_row_stride, k, k_row_stride, cand, prior, a_out,

@@ -119,6 +119,38 @@ def test_score_host_validation(case, want):
     assert e2s.e2s_status_string(st) == want
 
 
+@pytest.mark.parametrize("case,want", [
+    ("null_lse", "E2S_ERR_INVALID_ARG"),
+    ("misaligned_lse", "E2S_ERR_ALIGNMENT"),
+    ("eq1", "E2S_ERR_UNSUPPORTED"),
+    ("simt", "E2S_ERR_UNSUPPORTED"),
+    ("misaligned_q", "E2S_ERR_ALIGNMENT"),
+])
+def test_score_lse_host_validation(case, want):
+    """e2s_score_lse / e2s_decide_lse: the text rows' lse is required, 4-byte
+    aligned, and only the causal-probability score on the tcgen05 path uses it."""
+    e2s = _lib()
+    lay = _layout(e2s)
+    par = e2s.params()
+    ws, wsb = 0x100000, 1 << 20
+    q, k, qs, ks, lse = 0x200000, 0x300000, 32 * 128, 32 * 128, 0x500000
+    if case == "null_lse":
+        lse = None
+    elif case == "misaligned_lse":
+        lse = 0x500002
+    elif case == "eq1":
+        par = e2s.params(score_mode=e2s.E2S_SCORE_EQ1)
+    elif case == "simt":
+        par = e2s.params(flags=e2s.E2S_SIMT_SCORE)
+    elif case == "misaligned_q":
+        q = 0x200008
+    st = e2s.e2s_score_lse(lay, par, q, qs, k, ks, lse, 0x400000, ws, wsb, None)
+    assert e2s.e2s_status_string(st) == want
+    st = e2s.e2s_decide_lse(lay, par, q, qs, k, ks, lse, None, None, 0x400000, None, 0x600000,
+                            0x700000, 0x800000, 0x900000, 64, 0xA00000, None, ws, wsb, None)
+    assert e2s.e2s_status_string(st) == want
+
+
 def test_compact_host_validation():
     e2s = _lib()
     lay = _layout(e2s, sum_T=643, sum_vis=576)

@@ -83,3 +83,16 @@ def test_topk_tie_break_by_higher_index_is_caught():
     bad = np.sort(np.lexsort((-idx, -q))[:2])
     assert orc.topk(q, 2).tolist() == [0, 1]
     assert bad.tolist() != [0, 1]
+
+
+def test_lse_prefix_off_by_one_is_caught():
+    """A normaliser that stops one key short of the row's own position fails
+    the library logsumexp pin of causal_row_lse."""
+    from scipy.special import logsumexp
+    r = np.random.default_rng(13)
+    Q, K = r.normal(size=(3, 8)), r.normal(size=(10, 8))
+    logits = Q @ K.T / math.sqrt(8)
+    want = np.array([logsumexp(logits[t, :4 + t + 1]) for t in range(3)])
+    bad = np.array([logsumexp(logits[t, :4 + t]) for t in range(3)])
+    assert np.allclose(orc.causal_row_lse(Q, K, 4), want, atol=1e-12)
+    assert not np.allclose(bad, want, atol=1e-6)

@@ -375,3 +375,33 @@ def test_ds_generic_three_element_frame_example():
     assert m[frozenset({C})] == pytest.approx(0.3 / 0.7)
     assert ds.belief(m, frozenset({A, B})) == pytest.approx(0.4 / 0.7)
     assert ds.plausibility(m, frozenset({B})) == pytest.approx(0.2 / 0.7)
+
+
+def test_causal_row_lse_matches_library_logsumexp():
+    """Sec. 3.1: each text row's normaliser over its causal prefix, against
+    scipy's logsumexp of the visible logits taken row by row."""
+    from scipy.special import logsumexp
+    r = np.random.default_rng(11)
+    Q = r.normal(size=(5, 16))
+    K = r.normal(size=(12, 16))
+    lse = orc.causal_row_lse(Q, K, 6)
+    for t in range(5):
+        vis = [float(Q[t] @ K[j]) / 4.0 for j in range(6 + t + 1)]
+        assert abs(lse[t] - logsumexp(vis)) < 1e-12
+
+
+def test_causal_row_lse_reconstructs_attention_rows():
+    """exp(logit - lse) over the visible prefix is the causal softmax row, and
+    a row that sees a single key has lse equal to that key's logit."""
+    r = np.random.default_rng(12)
+    Q = r.normal(size=(4, 8))
+    K = r.normal(size=(9, 8))
+    lse = orc.causal_row_lse(Q, K, 5)
+    P = orc.causal_attention_rows(Q, K, 5)
+    logits = Q @ K.T / np.sqrt(8)
+    for t in range(4):
+        n = 5 + t + 1
+        assert np.allclose(np.exp(logits[t, :n] - lse[t]), P[t, :n], atol=1e-14)
+        assert np.all(P[t, n:] == 0)
+    one = orc.causal_row_lse(Q[:1], K, 0)
+    assert abs(one[0] - logits[0, 0]) < 1e-14
