@@ -383,6 +383,6 @@ const char* e2s_status_string(e2s_status s) {
   return "E2S_ERR_UNKNOWN";
 }
 
-int32_t e2s_version(void) { return 100; }
+int32_t e2s_version(void) { return 101; }
 
 }  // extern "C"

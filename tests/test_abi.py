@@ -57,7 +57,7 @@ def test_workspace_size_and_versions():
     # status word, one float4 per (image, layer, head), 64 cell keys + a counter per image
     assert n == 256 + ((1 * 2 * 32 * 16 + 255) // 256) * 256 + ((1 * 129 * 4 + 255) // 256) * 256
     assert e2s.e2s_workspace_size(_layout(e2s, d=64), e2s.params()) == 0
-    assert e2s.e2s_version() == 100
+    assert e2s.e2s_version() == 101
     assert e2s.e2s_status_string(e2s.E2S_ERR_TIMEOUT) == "E2S_ERR_TIMEOUT"
     assert e2s.e2s_status_string(99) == "E2S_ERR_UNKNOWN"
 
