@@ -383,6 +383,8 @@ def run_ours(args, world, rank, local):
         stream.synchronize()
         e2s.check(dec.status(stream), "device status after e2s_score_lse")
         lse_graph = capture([lse_call])
+        step_lse_graph = capture([lambda: dec.prune(q, k, src, dst, pos, stream=stream,
+                                                    lse=lse_dev)])
     launches_per_step = 3   # score, evidence/fusion/Top-K, compaction
 
     def run(gx):
@@ -412,6 +414,7 @@ def run_ours(args, world, rank, local):
             stage_ms = {name: [run(gx) for _ in range(n_stage)]
                         for name, gx in zip(stages, stage_graphs)}
             lse_ms = [run(lse_graph) for _ in range(n_stage)]
+            step_lse_ms = [run(step_lse_graph) for _ in range(n_stage)]
         if world > 1:
             torch.distributed.barrier()
         e2s.check(dec.status(stream), "device status after timing")
@@ -513,7 +516,8 @@ def run_ours(args, world, rank, local):
                     "from the layer's attention pass; streams only the visual key tiles",
             "us": statistics.mean(lse_ms) * 1e3,
             "algorithmic_bytes": bytes_lse,
-            "GB/s": bytes_lse / (statistics.mean(lse_ms) * 1e-3) / 1e9},
+            "GB/s": bytes_lse / (statistics.mean(lse_ms) * 1e-3) / 1e9,
+            "step_us": statistics.mean(step_lse_ms) * 1e3},
         "gpu_launches": launches_per_step * args.steps,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},

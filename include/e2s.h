@@ -197,6 +197,19 @@ e2s_status e2s_prune(const e2s_layout* layout, const e2s_params* params,
                      const int64_t* row_bytes, int32_t* pos_ids_out,
                      void* ws, size_t ws_bytes, void* stream);
 
+/* e2s_prune with its score taken as e2s_score_lse takes it (lse_text
+ * required, same restrictions). */
+e2s_status e2s_prune_lse(const e2s_layout* layout, const e2s_params* params,
+                         const void* q_text, int64_t q_row_stride,
+                         const void* k, int64_t k_row_stride, const float* lse_text,
+                         const int32_t* cand, const float* prior, float* a_out,
+                         float* mass_out, float* fused_out, float* q_out,
+                         const int32_t* keep_count, const int32_t* keep_off, int32_t sum_keep,
+                         int32_t* keep_idx, float* q_tilde_out,
+                         int32_t n_tensors, const void* const* src, void* const* dst,
+                         const int64_t* row_bytes, int32_t* pos_ids_out,
+                         void* ws, size_t ws_bytes, void* stream);
+
 /* Evidence and fusion (Sec. 4.1-4.2, Eqs. 8-19; Algorithm 1 inner loops).
  *   a          fp32 [L][H][sum_vis] from e2s_score.
  *   cand       nullable int32 [sum_vis]: original raster index of visual slot n

@@ -176,6 +176,33 @@ e2s_status check_compact_args(const e2s_layout* layout, const int32_t* keep_idx,
   return E2S_OK;
 }
 
+// e2s_prune / e2s_prune_lse (lse_text nullable here).
+e2s_status prune_impl(const e2s_layout* layout, const e2s_params* params,
+                      const void* q_text, int64_t q_row_stride, const void* k,
+                      int64_t k_row_stride, const float* lse_text, const int32_t* cand,
+                      const float* prior, float* a_out, float* mass_out, float* fused_out,
+                      float* q_out, const int32_t* keep_count, const int32_t* keep_off,
+                      int32_t sum_keep, int32_t* keep_idx, float* q_tilde_out,
+                      int32_t n_tensors, const void* const* src, void* const* dst,
+                      const int64_t* row_bytes, int32_t* pos_ids_out, void* ws,
+                      size_t ws_bytes, void* stream) {
+  E2S_TRY(check_decide_args(layout, params, q_text, q_row_stride, k, k_row_stride, prior, a_out,
+                            mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
+                            ws, ws_bytes));
+  E2S_TRY(check_compact_args(layout, keep_idx, keep_off, sum_keep, n_tensors, src, dst,
+                             row_bytes));
+  if (lse_text != nullptr) E2S_TRY(check_lse_args(layout, params, lse_text));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  E2S_TRY(run_decide(layout, params, q_text, q_row_stride, k, k_row_stride, cand, prior, a_out,
+                     mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
+                     q_tilde_out, ws, st, lse_text));
+  if (n_tensors == 0 && !pos_ids_out) return E2S_OK;
+  // the score kernel is an ordinary launch: it starts after all earlier work on
+  // the stream, so the sources are complete before the compaction may start
+  return from_cuda(launch_compact(layout_args(layout), keep_idx, keep_off, sum_keep, n_tensors,
+                                  src, dst, row_bytes, pos_ids_out, status_word(ws), st, 1));
+}
+
 }  // namespace
 }  // namespace e2s
 
@@ -251,20 +278,26 @@ e2s_status e2s_prune(const e2s_layout* layout, const e2s_params* params, const v
                      float* q_tilde_out, int32_t n_tensors, const void* const* src,
                      void* const* dst, const int64_t* row_bytes, int32_t* pos_ids_out, void* ws,
                      size_t ws_bytes, void* stream) {
-  E2S_TRY(check_decide_args(layout, params, q_text, q_row_stride, k, k_row_stride, prior, a_out,
-                            mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
-                            ws, ws_bytes));
-  E2S_TRY(check_compact_args(layout, keep_idx, keep_off, sum_keep, n_tensors, src, dst,
-                             row_bytes));
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  E2S_TRY(run_decide(layout, params, q_text, q_row_stride, k, k_row_stride, cand, prior, a_out,
-                     mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
-                     q_tilde_out, ws, st));
-  if (n_tensors == 0 && !pos_ids_out) return E2S_OK;
-  // the score kernel is an ordinary launch: it starts after all earlier work on
-  // the stream, so the sources are complete before the compaction may start
-  return from_cuda(launch_compact(layout_args(layout), keep_idx, keep_off, sum_keep, n_tensors,
-                                  src, dst, row_bytes, pos_ids_out, status_word(ws), st, 1));
+  return prune_impl(layout, params, q_text, q_row_stride, k, k_row_stride, nullptr, cand, prior,
+                    a_out, mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
+                    q_tilde_out, n_tensors, src, dst, row_bytes, pos_ids_out, ws, ws_bytes,
+                    stream);
+}
+
+e2s_status e2s_prune_lse(const e2s_layout* layout, const e2s_params* params,
+                         const void* q_text, int64_t q_row_stride, const void* k,
+                         int64_t k_row_stride, const float* lse_text, const int32_t* cand,
+                         const float* prior, float* a_out, float* mass_out, float* fused_out,
+                         float* q_out, const int32_t* keep_count, const int32_t* keep_off,
+                         int32_t sum_keep, int32_t* keep_idx, float* q_tilde_out,
+                         int32_t n_tensors, const void* const* src, void* const* dst,
+                         const int64_t* row_bytes, int32_t* pos_ids_out, void* ws,
+                         size_t ws_bytes, void* stream) {
+  if (!lse_text) return E2S_ERR_INVALID_ARG;
+  return prune_impl(layout, params, q_text, q_row_stride, k, k_row_stride, lse_text, cand, prior,
+                    a_out, mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
+                    q_tilde_out, n_tensors, src, dst, row_bytes, pos_ids_out, ws, ws_bytes,
+                    stream);
 }
 
 e2s_status e2s_fuse(const e2s_layout* layout, const e2s_params* params, const float* a,

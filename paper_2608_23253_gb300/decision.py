@@ -163,10 +163,19 @@ class Decision:
     def prune(self, q_text: torch.Tensor, k: torch.Tensor, src: Sequence[torch.Tensor],
               dst: Sequence[torch.Tensor], pos_ids: Optional[torch.Tensor] = None,
               prior: Optional[torch.Tensor] = None, cand: Optional[torch.Tensor] = None,
-              stream=None) -> None:
-        """The whole pruning step (e2s_prune): decide, then compact src into dst."""
+              stream=None, lse: Optional[torch.Tensor] = None) -> None:
+        """The whole pruning step (e2s_prune): decide, then compact src into dst
+        (e2s_prune_lse when the text rows' attention lse is given)."""
         b = self.batch
         row_bytes = [t.stride(0) * t.element_size() for t in src]
+        if lse is not None:
+            e2s.check(e2s.e2s_prune_lse(b.layout, self.params, q_text, b.H * b.d, k,
+                                        b.H_kv * b.d, lse, cand, prior, self.a, self.mass,
+                                        self.fused, self.q, self.keep_count, self.keep_off,
+                                        self.sum_keep, self.keep_idx, self.q_tilde, len(src), src,
+                                        dst, row_bytes, pos_ids, self.ws, self.ws_bytes, stream),
+                      "e2s_prune_lse")
+            return
         e2s.check(e2s.e2s_prune(b.layout, self.params, q_text, b.H * b.d, k, b.H_kv * b.d, cand,
                                 prior, self.a, self.mass, self.fused, self.q, self.keep_count,
                                 self.keep_off, self.sum_keep, self.keep_idx, self.q_tilde,

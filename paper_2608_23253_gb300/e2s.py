@@ -81,6 +81,9 @@ _SIGS = {
     "e2s_prune": (ctypes.c_int, [_LP, _PP, _vp, _i64, _vp, _i64, _vp, _vp, _vp, _vp, _vp, _vp,
                                   _vp, _vp, _i32, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _sz,
                                   _vp]),
+    "e2s_prune_lse": (ctypes.c_int, [_LP, _PP, _vp, _i64, _vp, _i64, _vp, _vp, _vp, _vp, _vp,
+                                      _vp, _vp, _vp, _vp, _i32, _vp, _vp, _i32, _vp, _vp, _vp,
+                                      _vp, _vp, _sz, _vp]),
     "e2s_fuse": (ctypes.c_int, [_LP, _PP, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "e2s_fuse_select": (ctypes.c_int, [_LP, _PP, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _i32,
                                         _vp, _vp, _vp, _sz, _vp]),
@@ -169,6 +172,21 @@ def _addr_arrays(src, dst, row_bytes, n):
     rb_a = (ctypes.c_int64 * max(n, 1))(*[int(x) for x in row_bytes])
     return (ctypes.cast(src_a, ctypes.c_void_p), ctypes.cast(dst_a, ctypes.c_void_p),
             ctypes.cast(rb_a, ctypes.c_void_p), (src_a, dst_a, rb_a))
+
+
+def e2s_prune_lse(layout, params_, q_text, q_row_stride, k, k_row_stride, lse_text, cand, prior,
+                  a_out, mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
+                  q_tilde_out, n_tensors, src, dst, row_bytes, pos_ids_out, ws, ws_bytes,
+                  stream=None) -> int:
+    """src/dst: sequences of tensors or addresses; row_bytes: sequence of ints."""
+    n = int(n_tensors)
+    s_p, d_p, r_p, _keep = _addr_arrays(src, dst, row_bytes, n)
+    return lib.e2s_prune_lse(_ref(layout), _ref(params_), _ptr(q_text), q_row_stride, _ptr(k),
+                             k_row_stride, _ptr(lse_text), _ptr(cand), _ptr(prior), _ptr(a_out),
+                             _ptr(mass_out), _ptr(fused_out), _ptr(q_out), _ptr(keep_count),
+                             _ptr(keep_off), sum_keep, _ptr(keep_idx), _ptr(q_tilde_out), n,
+                             s_p, d_p, r_p, _ptr(pos_ids_out), _ptr(ws), ws_bytes,
+                             _stream(stream))
 
 
 def e2s_prune(layout, params_, q_text, q_row_stride, k, k_row_stride, cand, prior, a_out,

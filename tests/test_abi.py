@@ -149,6 +149,10 @@ def test_score_lse_host_validation(case, want):
     st = e2s.e2s_decide_lse(lay, par, q, qs, k, ks, lse, None, None, 0x400000, None, 0x600000,
                             0x700000, 0x800000, 0x900000, 64, 0xA00000, None, ws, wsb, None)
     assert e2s.e2s_status_string(st) == want
+    st = e2s.e2s_prune_lse(lay, par, q, qs, k, ks, lse, None, None, 0x400000, None, 0x600000,
+                           0x700000, 0x800000, 0x900000, 64, 0xA00000, None, 0, [], [], [], None,
+                           ws, wsb, None)
+    assert e2s.e2s_status_string(st) == want
 
 
 def test_compact_host_validation():

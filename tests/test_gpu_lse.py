@@ -62,3 +62,34 @@ def test_decide_lse_matches_oracle(case):
     parity.check_topk_of_own_scores(gpu["keep"], gpu["q_tilde"], inp.n_vis, inp.keep)
     for b in parity.clear_margin_images(ref, inp.n_vis, inp.keep):
         assert np.array_equal(gpu["keep"][b], ref["keep"][b])
+
+
+@pytest.mark.parametrize("case", ["llava-b1", "qwen2vl-gqa-b4"])
+def test_prune_lse_compaction_bit_exact(case):
+    """e2s_prune_lse: the decision from the attention lse, then every output
+    row is the oracle's compaction of the keep set the GPU chose, bit for bit."""
+    from paper_2608_23253_gb300.decision import bf16_tensor
+    cfg, batch = CASES[case]
+    inp = config_inputs(cfg, batch, None, True)
+    _, dec, q, k, lse = _setup(case)
+    ref = config_oracle(cfg, batch, None, "causal")
+    dev = device()
+    L = inp.spec.L
+    host = [inp.hidden] + [inp.k[l].reshape(inp.k.shape[1], -1) for l in range(L)] + \
+           [inp.v[l].reshape(inp.v.shape[1], -1) for l in range(L)]
+    src = [bf16_tensor(x, dev) for x in host]
+    R = dec.out_rows()
+    dst = [torch.full((R, t.shape[1]), -1, dtype=t.dtype, device=dev) for t in src]
+    pos = torch.full((R,), -7, dtype=torch.int32, device=dev)
+    dec.prune(q, k, src, dst, pos, lse=lse)
+    torch.cuda.synchronize()
+    assert dec.status() == 0
+    keep = dec.keep_lists()
+    parity.assert_close("a", dec.a.cpu().numpy(), ref["a"])
+    parity.check_selection(keep, dec.q_tilde.cpu().numpy(), ref["q"], inp.n_vis, inp.grid_h,
+                           inp.grid_w, inp.keep, 0.1, 4)
+    for d_, h_ in zip(dst, host):
+        want = orc.compact(h_, inp.n_sys, inp.n_vis, inp.n_text, keep)
+        assert np.array_equal(d_.cpu().view(torch.int16).numpy().view(np.uint16), want)
+    assert np.array_equal(pos.cpu().numpy(),
+                          orc.position_ids(inp.n_sys, inp.n_vis, inp.n_text, keep))
