@@ -22,12 +22,31 @@ CASES = {"llava-b1": (1, None), "llava-ragged-b6": (2, 6), "qwen2vl-gqa-b4": (3,
          "highres-b2": (4, 2)}
 
 
+def _inputs(case):
+    if case == "gqa-stack4":
+        # 28 query / 4 kv heads, at most 32 text rows: four heads per unit
+        from paper_2608_23253_gb300 import synth
+        from paper_2608_23253_gb300.synth import ImageSpec
+        ims = [ImageSpec(35, 24, 24, 32, 40, 3, 64), ImageSpec(3, 13, 17, 9, 12, 2, 50),
+               ImageSpec(0, 30, 20, 1, 30, 3, 66)]
+        return synth.make_inputs(synth.custom_spec("lse", ims, L=2, H=28, H_kv=4, cfg_id=95),
+                                 with_payload=False)
+    cfg, batch = CASES[case]
+    return config_inputs(cfg, batch, None)
+
+
+def _reference(case, inp):
+    if case == "gqa-stack4":
+        from tests.gpu_helpers import run_oracle
+        return run_oracle(inp, "causal")
+    return config_oracle(*CASES[case], None, "causal")
+
+
 def _setup(case):
     from paper_2608_23253_gb300 import e2s
     from paper_2608_23253_gb300.decision import Batch, Decision, bf16_tensor
-    cfg, batch = CASES[case]
     dev = device()
-    inp = config_inputs(cfg, batch, None)
+    inp = _inputs(case)
     lse = orc.text_row_lse(inp.q_text, inp.k, inp.n_sys, inp.n_vis, inp.n_text,
                            H_kv=inp.spec.H_kv)
     dec = Decision(Batch.from_inputs(inp, device=dev), inp.keep, e2s.params())
@@ -36,20 +55,20 @@ def _setup(case):
     return inp, dec, q, k, torch.as_tensor(lse.astype(np.float32), device=dev)
 
 
-@pytest.mark.parametrize("case", sorted(CASES))
+@pytest.mark.parametrize("case", sorted(CASES) + ["gqa-stack4"])
 def test_score_lse_matches_oracle(case):
     inp, dec, q, k, lse = _setup(case)
-    ref = config_oracle(*CASES[case], None, "causal")
+    ref = _reference(case, inp)
     dec.score(q, k, lse=lse)
     torch.cuda.synchronize()
     assert dec.status() == 0
     parity.assert_close("a", dec.a.cpu().numpy(), ref["a"])
 
 
-@pytest.mark.parametrize("case", sorted(CASES))
+@pytest.mark.parametrize("case", sorted(CASES) + ["gqa-stack4"])
 def test_decide_lse_matches_oracle(case):
     inp, dec, q, k, lse = _setup(case)
-    ref = config_oracle(*CASES[case], None, "causal")
+    ref = _reference(case, inp)
     dec.decide(q, k, lse=lse)
     torch.cuda.synchronize()
     assert dec.status() == 0
