@@ -51,6 +51,24 @@ def test_config_shapes(cfg):
         assert {im.n_vis: im.n_salient for im in spec.images} == {2304: 115, 4096: 205}
 
 
+@pytest.mark.parametrize("ratio", [1 / 3, 2 / 9])
+def test_qwen2vl_dynamic_grid_spec(ratio):
+    """Sec. 4.5's reduction ratios on merged-patch grids of any shape."""
+    spec = synth.config_spec(3, keep_ratio=ratio, dynamic_grids=True)
+    again = synth.config_spec(3, keep_ratio=ratio, dynamic_grids=True)
+    assert [(i.grid_h, i.grid_w) for i in spec.images] == \
+        [(i.grid_h, i.grid_w) for i in again.images]
+    assert (spec.B, spec.H, spec.H_kv, spec.L) == (16, 28, 4, 3)
+    for im in spec.images:
+        assert 12 <= im.grid_h <= 48 and 12 <= im.grid_w <= 48 and im.n_vis <= 1296
+        assert im.keep == int(np.round(ratio * im.n_vis))
+        assert im.n_text == 64
+    assert any(im.grid_h % 4 or im.grid_w % 4 for im in spec.images)
+    # the fixed-grid configuration is unchanged by the new options' defaults
+    assert [(i.grid_h, i.grid_w, i.keep) for i in synth.config_spec(3).images] == \
+        [(i.grid_h, i.grid_w, i.keep) for i in synth.config_spec(3, keep_ratio=None).images]
+
+
 def test_generator_deterministic_and_planted():
     spec = synth.config_spec(1)
     a = synth.make_inputs(spec, with_payload=False)
