@@ -59,6 +59,43 @@ constexpr uint64_t kWaitNs = 1000000000ull;
 constexpr uint64_t kWaitNsAfterFault = 1000000ull;
 constexpr float kLog2e = 1.4426950408889634f;
 
+// Two fp32 lanes in one 64-bit register: packed FMA and add (fma.rn.f32x2,
+// add.rn.f32x2), each lane rounded exactly as fmaf / + would round it.
+__device__ __forceinline__ uint64_t f2pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2unpack(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+// sum over 16 logits of exp2(x * s + n_j), even and odd lanes accumulated
+// separately from (acc_even, acc_odd), then added
+__device__ __forceinline__ float exp2_sum16(const float (&x)[16], float s, const float (&n)[16],
+                                            float acc_even) {
+  const uint64_t s2 = f2pack(s, s);
+  uint64_t acc = f2pack(acc_even, 0.f);
+#pragma unroll
+  for (int j = 0; j < 16; j += 2) {
+    float t0, t1;
+    f2unpack(ffma2(f2pack(x[j], x[j + 1]), s2, f2pack(n[j], n[j + 1])), t0, t1);
+    acc = fadd2(acc, f2pack(fast_ex2(t0), fast_ex2(t1)));
+  }
+  float a0, a1;
+  f2unpack(acc, a0, a1);
+  return a0 + a1;
+}
+
 struct StreamArgs {
   LayoutArgs la;
   int mode;
@@ -86,7 +123,7 @@ __host__ __device__ inline SPlan stream_plan(int stages) {
   s.bars = s.k + (uint32_t)stages * kTileBytes;         // mbarriers, see the kernel
   s.slot = s.bars + 8u * (uint32_t)(2 + 2 * kMaxStages + 4 + kMaxBatch + 1);
   s.ms = (s.slot + 16u + 15u) & ~15u;                   // [4][128] float2 (max, sum)
-  s.lse = s.ms + 4u * kRows * 8u;                       // [128] float lse per text row
+  s.lse = s.ms + 4u * kRows * 8u;                       // [128] float -lse per text row
   s.cps = s.lse + kRows * 4u;                           // [2][8 chunks][128 keys] partials
   s.red = s.cps + 2u * 8u * kTileKeys * 4u;             // [4 heads][4] float4 statistics
   s.total = s.red + 16u * 16u;
@@ -184,7 +221,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* b_done = b_full + kMaxBatch;   // batch sweep 2 read: TMEM free again
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + plan.slot);
   float2* ms = reinterpret_cast<float2*>(smem + plan.ms);
-  float* lse_s = reinterpret_cast<float*>(smem + plan.lse);
+  float* nlse = reinterpret_cast<float*>(smem + plan.lse);   // -lse per text row
   float* cps = reinterpret_cast<float*>(smem + plan.cps);
   float4* red = reinterpret_cast<float4*>(smem + plan.red);
 
@@ -406,13 +443,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
               for (int jj = 1; jj < 16; ++jj) cmax = fmaxf(cmax, x[jj]);
               const float mnew = fmaxf(m, cmax * p.scale_log2);
-              float acc0 = ssum * fast_ex2(m - mnew), acc1 = 0.f;
+              float nm[16];
 #pragma unroll
-              for (int jj = 0; jj < 16; jj += 2) {
-                acc0 += fast_ex2(fmaf(x[jj], p.scale_log2, -mnew));
-                acc1 += fast_ex2(fmaf(x[jj + 1], p.scale_log2, -mnew));
-              }
-              ssum = acc0 + acc1;
+              for (int jj = 0; jj < 16; ++jj) nm[jj] = -mnew;
+              ssum = exp2_sum16(x, p.scale_log2, nm, ssum * fast_ex2(m - mnew));
               m = mnew;
             } else if (key0 <= lim && key0 + 15 >= 0) {   // key 0 or the row's last key inside
               float cmax = kNegBig;
@@ -438,9 +472,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       // per text row for sweep 2 (or taken from the caller's attention pass)
       if (causal && p.lse_in != nullptr) {
         if (cg == 0 && (!SPLIT || lrow < kRows / 2))
-          lse_s[lrow] = tvalid ? __ldg(p.lse_in + ((size_t)g.l * la.H + g.h + hs) * la.sum_text +
+          nlse[lrow] = tvalid ? -__ldg(p.lse_in + ((size_t)g.l * la.H + g.h + hs) * la.sum_text +
                                        g.x0 + t) * kLog2e
-                               : kNegBig;
+                              : -kNegBig;
         ptx::named_bar(1, kEpiThreads);
       } else if (causal) {
         ms[cg * kRows + lrow] = make_float2(m, ssum);
@@ -459,7 +493,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float2 v = part(c);
           L += v.y * fast_ex2(v.x - M);
         }
-        if (cg == 0 && (!SPLIT || lrow < kRows / 2)) lse_s[lrow] = L > 0.f ? M + __log2f(L) : kNegBig;
+        if (cg == 0 && (!SPLIT || lrow < kRows / 2))
+          nlse[lrow] = L > 0.f ? -(M + __log2f(L)) : -kNegBig;
         ptx::named_bar(1, kEpiThreads);
       }
       // ---- sweep 2: accumulator D[key][column], keys on the lanes, so each
@@ -488,17 +523,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int c = 0; c < nch; ++c) {
               float x[16];
               ptx::tmem_ld16(tb + (uint32_t)(c * 16), x);
-              const float4* l4 = reinterpret_cast<const float4*>(lse_s + c * 16);
+              const float4* l4 = reinterpret_cast<const float4*>(nlse + c * 16);
               float s0 = 0.f, s1 = 0.f;
               if (c * 16 + 15 < g.NT) {
+                float nl[16];
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                   const float4 v = l4[q];
-                  s0 += fast_ex2(fmaf(x[4 * q], p.scale_log2, -v.x));
-                  s1 += fast_ex2(fmaf(x[4 * q + 1], p.scale_log2, -v.y));
-                  s0 += fast_ex2(fmaf(x[4 * q + 2], p.scale_log2, -v.z));
-                  s1 += fast_ex2(fmaf(x[4 * q + 3], p.scale_log2, -v.w));
+                  nl[4 * q] = v.x; nl[4 * q + 1] = v.y; nl[4 * q + 2] = v.z; nl[4 * q + 3] = v.w;
                 }
+                s0 = exp2_sum16(x, p.scale_log2, nl, 0.f);
               } else {
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
@@ -507,7 +541,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                   for (int i = 0; i < 4; ++i)
                     if (c * 16 + 4 * q + i < g.NT)
-                      s0 += fast_ex2(fmaf(x[4 * q + i], p.scale_log2, -lv[i]));
+                      s0 += fast_ex2(fmaf(x[4 * q + i], p.scale_log2, lv[i]));
                 }
               }
               a += s0 + s1;
@@ -541,7 +575,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::tmem_ld16(tmem + lane_base + (uint32_t)(buf * kTileKeys + c * 16), x);
             float acc0 = 0.f, acc1 = 0.f;
             if (causal) {
-              const float4* l4 = reinterpret_cast<const float4*>(lse_s + c * 16);
+              const float4* l4 = reinterpret_cast<const float4*>(nlse + c * 16);
               float lv[16];
 #pragma unroll
               for (int q = 0; q < 4; ++q) {
@@ -549,15 +583,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 lv[4 * q] = v.x; lv[4 * q + 1] = v.y; lv[4 * q + 2] = v.z; lv[4 * q + 3] = v.w;
               }
               if (ct + 15 < g.NT) {
-#pragma unroll
-                for (int jj = 0; jj < 16; jj += 2) {
-                  acc0 += fast_ex2(fmaf(x[jj], p.scale_log2, -lv[jj]));
-                  acc1 += fast_ex2(fmaf(x[jj + 1], p.scale_log2, -lv[jj + 1]));
-                }
+                acc0 = exp2_sum16(x, p.scale_log2, lv, 0.f);
               } else {
 #pragma unroll
                 for (int jj = 0; jj < 16; ++jj)
-                  if (ct + jj < g.NT) acc0 += fast_ex2(fmaf(x[jj], p.scale_log2, -lv[jj]));
+                  if (ct + jj < g.NT) acc0 += fast_ex2(fmaf(x[jj], p.scale_log2, lv[jj]));
               }
             } else {
 #pragma unroll
@@ -615,7 +645,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         p.stats[((size_t)g.b * la.L + g.l) * la.H + g.h + et] = stats_entry(S, M, E);
       }
-      // ms, lse_s, cps and red are rewritten by the next unit only after this barrier
+      // ms, nlse, cps and red are rewritten by the next unit only after this barrier
       ptx::named_bar(1, kEpiThreads);
     }
   }
