@@ -424,37 +424,68 @@ def run_ours(args, world, rank, local):
                    for x in (inp.q_text, inp.k, inp.v, inp.hidden)]
         dev_in = [q, k, v, hid]
         h2d = sum(t.numel() * t.element_size() for t in host_in)
-        out_keep = torch.empty(dec.keep_idx.numel(), dtype=torch.int32).pin_memory()
-        out_pos = torch.empty(R, dtype=torch.int32).pin_memory()
-        d2h = out_keep.numel() * 4 + out_pos.numel() * 4
-        # Q and K are copied first; V and the hidden states, which only the
-        # compaction reads, follow on a second stream while e2s_decide runs
-        side = torch.cuda.Stream(device=dev)
-        ev_qk, ev_vh = torch.cuda.Event(), torch.cuda.Event()
-        e2e_ms = []
-        for it in range(args.warmup + args.steps):
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            for hsrc, ddst in zip(host_in[:2], dev_in[:2]):
-                ddst.view(torch.int16).view(-1).copy_(hsrc.view(-1), non_blocking=True)
-            ev_qk.record(stream)
-            side.wait_event(ev_qk)
-            with torch.cuda.stream(side):
-                for hsrc, ddst in zip(host_in[2:], dev_in[2:]):
+        # Pipelined over two input slots: a copy stream uploads each step's
+        # inputs (Q and K first; V and the hidden states, which only the
+        # compaction reads, after them) while the compute stream runs the
+        # previous step; a slot is reused once the step that read it is done
+        slots = [dict(dev_in=dev_in, dec=dec, g_dec=stage_graphs[1][0],
+                      g_cmp=stage_graphs[2][0], pos=pos)]
+        q1, k1, v1, hid1 = (t.clone() for t in dev_in)
+        dec1 = Decision(batch, inp.keep, e2s.params())
+        src1 = [hid1] + [k1[l].view(batch.sum_T, kv_rows) for l in range(s.L)] + \
+               [v1[l].view(batch.sum_T, kv_rows) for l in range(s.L)]
+        dst1 = [torch.empty_like(t) for t in dst]
+        pos1 = torch.empty_like(pos)
+        dec1.decide(q1, k1, stream=stream)
+        dec1.compact(src1, dst1, pos1, stream=stream)
+        stream.synchronize()
+        e2s.check(dec1.status(stream), "device status after the second slot's warm-up")
+        # capture() returns (graph, start event, end event); the events stay
+        # referenced for as long as the graph that records them
+        cap_dec1 = capture([lambda: dec1.decide(q1, k1, stream=stream)])
+        cap_cmp1 = capture([lambda: dec1.compact(src1, dst1, pos1, stream=stream)])
+        slots.append(dict(dev_in=[q1, k1, v1, hid1], dec=dec1, g_dec=cap_dec1[0],
+                          g_cmp=cap_cmp1[0], keep_alive=(cap_dec1, cap_cmp1), pos=pos1))
+        for sl in slots:
+            sl["out_keep"] = torch.empty(dec.keep_idx.numel(), dtype=torch.int32).pin_memory()
+            sl["out_pos"] = torch.empty(R, dtype=torch.int32).pin_memory()
+            sl["ev_qk"], sl["ev_vh"], sl["ev_done"] = (torch.cuda.Event() for _ in range(3))
+        d2h = slots[0]["out_keep"].numel() * 4 + slots[0]["out_pos"].numel() * 4
+        copy_s = torch.cuda.Stream(device=dev)
+
+        def e2e_step(it):
+            sl = slots[it % 2]
+            copy_s.wait_event(sl["ev_done"])
+            with torch.cuda.stream(copy_s):
+                for j, (hsrc, ddst) in enumerate(zip(host_in, sl["dev_in"])):
                     ddst.view(torch.int16).view(-1).copy_(hsrc.view(-1), non_blocking=True)
-                ev_vh.record(side)
-            stage_graphs[1][0].replay()   # e2s_decide: score, evidence / fusion / Top-K
-            stream.wait_event(ev_vh)
-            stage_graphs[2][0].replay()   # e2s_compact
-            out_keep.copy_(dec.keep_idx, non_blocking=True)
-            out_pos.copy_(pos, non_blocking=True)
-            e1.record(stream)
-            e1.synchronize()
-            if it >= args.warmup:
-                e2e_ms.append(e0.elapsed_time(e1))
-        e2s.check(dec.status(stream), "device status after the end-to-end loop")
-        if not torch.equal(out_keep, dec.keep_idx.cpu()):
-            raise RuntimeError("end-to-end keep list differs from the device result")
+                    if j == 1:
+                        sl["ev_qk"].record(copy_s)
+                sl["ev_vh"].record(copy_s)
+            stream.wait_event(sl["ev_qk"])
+            sl["g_dec"].replay()   # e2s_decide: score, evidence / fusion / Top-K
+            stream.wait_event(sl["ev_vh"])
+            sl["g_cmp"].replay()   # e2s_compact
+            sl["out_keep"].copy_(sl["dec"].keep_idx, non_blocking=True)
+            sl["out_pos"].copy_(sl["pos"], non_blocking=True)
+            sl["ev_done"].record(stream)
+
+        for it in range(args.warmup):
+            e2e_step(it)
+        torch.cuda.synchronize()
+        t_e0, t_e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t_e0.record(copy_s)
+        for it in range(args.warmup, args.warmup + args.steps):
+            e2e_step(it)
+        t_e1.record(stream)
+        t_e1.synchronize()
+        e2e_ms = [t_e0.elapsed_time(t_e1) / args.steps] * args.steps
+        for sl in slots:
+            e2s.check(sl["dec"].status(stream), "device status after the end-to-end loop")
+            if not torch.equal(sl["out_keep"], sl["dec"].keep_idx.cpu()):
+                raise RuntimeError("end-to-end keep list differs from the device result")
+        if not torch.equal(slots[0]["out_keep"], slots[1]["out_keep"]):
+            raise RuntimeError("the two input slots decided differently")
 
     total_ms, e2e_total, value, e2e_value = combine_ranks(
         sum(step_ms), sum(e2e_ms), batch.B * args.steps, world, dev)
