@@ -135,7 +135,9 @@ e2s_status e2s_score(const e2s_layout* layout, const e2s_params* params,
  * row normalisers.
  *   lse_text  fp32 [L][H][sum_text], device, 4-byte aligned:
  *             lse_text[(l*H + h)*sum_text + text_off[b] + t] for text row t of
- *             image b, query head h, layer l.  Its accuracy bounds that of a.
+ *             image b, query head h, layer l; finite for every text row.  Its
+ *             accuracy bounds that of a (a relative error e in exp(-lse)
+ *             scales a by 1 + e), so it should be float32-exact.
  * Other arguments, the results and the Eq. 8 statistics left in the workspace
  * are those of e2s_score.  E2S_ERR_UNSUPPORTED unless score_mode is
  * CAUSAL_PROB, E2S_SIMT_SCORE is clear and max_text <= 128. */
