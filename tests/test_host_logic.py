@@ -119,3 +119,20 @@ def test_multiply_high_division_is_exact():
             n = n[n < (1 << 17)]
             got = (n * np.uint64(m)) >> np.uint64(32)
             assert np.array_equal(got, n // np.uint64(d)), d
+
+
+def test_bench_attention_lse_matches_oracle():
+    """bench.py's stand-in for the attention pass's row lse (torch, float32)
+    against the oracle's float64 causal_row_lse, on the CPU."""
+    import bench
+    from oracle import e2s_oracle as orc
+    inp = synth.make_inputs(synth.custom_spec(
+        "lse", [synth.ImageSpec(35, 12, 12, 20, 10, 2, 30),
+                synth.ImageSpec(3, 5, 7, 9, 4, 0, 10)], L=2, H=8, H_kv=2, cfg_id=94),
+        with_payload=False)
+    q = torch.from_numpy(inp.q_text.view(np.int16)).view(torch.bfloat16)
+    k = torch.from_numpy(inp.k.view(np.int16)).view(torch.bfloat16)
+    got = bench.attention_lse(inp, q, k, torch.device("cpu")).numpy()
+    want = orc.text_row_lse(inp.q_text, inp.k, inp.n_sys, inp.n_vis, inp.n_text, H_kv=2)
+    assert got.shape == want.shape
+    assert np.abs(got - want).max() < 1e-4
