@@ -152,7 +152,7 @@ e2s_status e2s_score_lse(const e2s_layout* layout, const e2s_params* params,
  * a_out is required (it carries a[l][h][n] from the first launch to the
  * second).  The score kernel also leaves the Eq. 8 normalisation statistics
  * of every (image, layer, head) in the workspace, so the second kernel treats
- * every visual token independently (one warp per token) and the last CTA to
+ * every visual token independently (no cross-CTA reduction) and the last CTA to
  * finish an image runs that image's Top-K.  Results are identical to
  * e2s_score, e2s_fuse and e2s_select called in sequence, up to the rounding
  * order of the normalisation sums.  keep_count and keep_off are required;

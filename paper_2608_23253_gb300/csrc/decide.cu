@@ -1,13 +1,15 @@
 // Evidence, layer-wise fusion and selection of e2s_decide (Sec. 4.1-4.3,
 // Eqs. 8-23), token-parallel.  The normalisation statistics of Eq. 8 for
 // every (image, layer, head) were produced by the score kernel, so tokens are
-// independent here.  A CTA of 256 threads takes 64 visual tokens of one image:
+// independent here.  A CTA of 256 threads takes 64 visual tokens of one image
+// (16 when the batch is too small to fill the GPU with 64-token CTAs):
 //   1. the image's statistics and the CTA's a[l][h][token] values are copied
 //      into shared memory with asynchronous copies, all in flight at once;
-//   2. one thread per (token, layer) walks the H heads: supports p (Eq. 9),
-//      written back over the staged scores, p_bar, then the reliability terms
-//      of Eq. 10, rho and the layer mass (Eq. 11) -- independent iterations,
-//      no cross-thread reduction;
+//   2. one thread per (token, layer) walks the H heads (with 16-token CTAs,
+//      four lanes per (token, layer), each taking every fourth head, joined by
+//      two shuffles): supports p (Eq. 9), written back over the staged
+//      scores, p_bar, then the reliability terms of Eq. 10, rho and the layer
+//      mass (Eq. 11);
 //   3. one thread per token: Dempster combination of its layer masses in
 //      order (Eqs. 12-16), Pl and q (Eqs. 18-19), and its bid for its cell's
 //      representative (Eqs. 20-21);
