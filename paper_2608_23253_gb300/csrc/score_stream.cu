@@ -20,7 +20,9 @@
 //           P = exp2(s - lse_t) over the text rows of its column chunks, the
 //           chunk partials of a key are added in a fixed order through shared
 //           memory, and a[key] = sum_t P / N_T.
-// EQ1 mode has no sweep 1 and sums s / sqrt(d) / N_T in sweep 2.
+// EQ1 mode has no sweep 1 and sums s / sqrt(d) / N_T in sweep 2.  Neither has
+// CAUSAL_PROB when the caller supplies each text row's lse from the layer's
+// own attention pass (lse_in): sweep 2 alone then streams the visual tiles.
 // K tiles stream through a ring of as many stages as shared memory holds
 // (TMA producer warp; deep enough to cover the load latency), the accumulator
 // is double-buffered in TMEM (MMA warp), so loads, MMAs and the epilogue of
