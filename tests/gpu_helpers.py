@@ -69,11 +69,13 @@ def run_gpu(inp, mode: str = "causal", *, simt: bool = False, flags: int = 0, la
 def run_oracle(inp, mode: str = "causal", *, flags: int = 0, lam: float = 0.1, G: int = 4,
                keep=None, norm=None, prior=None, cand=None, grid_h=None, grid_w=None):
     p = orc.Params(lam=lam, G=G, score_mode=MODES[mode][1], norm_mode=norm, flags=flags)
-    return orc.decide(inp.q_text, inp.k, inp.n_sys, inp.n_vis, inp.n_text,
+    out = orc.decide(inp.q_text, inp.k, inp.n_sys, inp.n_vis, inp.n_text,
                       inp.grid_h if grid_h is None else grid_h,
                       inp.grid_w if grid_w is None else grid_w,
                       inp.keep if keep is None else keep, H_kv=inp.spec.H_kv, params=p,
                       prior=prior, cand=cand)
+    out["score_mode"] = p.score_mode
+    return out
 
 
 @functools.lru_cache(maxsize=None)

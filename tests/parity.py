@@ -2,7 +2,14 @@
 
 Tolerances (floating point): every float output -- a, masses, p_bar, fused
 masses, conflict K, q and q~ -- within max abs 1e-3 of the float64 oracle
-(bf16 inputs, fp32 accumulation on the GPU).
+(bf16 inputs, fp32 accumulation on the GPU).  Causal-probability scores are
+also held to an elementwise relative bound, A_REL: a token's a is about
+1/N_V (1.7e-3 on a 24 x 24 grid), the same size as the absolute tolerance, so
+that tolerance alone cannot see a wrong score.  Dropping one text row from the
+mean moves a by up to 2-3 % of its value on the LLaVA shapes, and a causal
+mask one key short by 0.16 % (tests/test_parity_bounds.py); the GPU's own
+error is about 1e-5 relative (fp32 sums of ex2.approx terms, relative error
+~2^-22 each).
 
 Discrete outputs, where floating point decides an integer:
   * cell representative b (Eqs. 20-21): where the oracle's best q in a cell
@@ -22,6 +29,7 @@ import numpy as np
 from oracle import e2s_oracle as orc
 
 TOL = 1e-3
+A_REL = 5e-4
 
 
 def max_err(got, want) -> float:
@@ -40,8 +48,22 @@ def assert_close(name, got, want, tol=TOL):
     return e
 
 
+def check_a(got, want, causal: bool, tol=TOL, rel=A_REL):
+    """a within the absolute tolerance, and for causal-probability scores
+    (strictly positive) within `rel` of each oracle value."""
+    e = assert_close("a", got, want, tol)
+    if causal and np.size(want):
+        g = np.asarray(got, dtype=np.float64)
+        w = np.asarray(want, dtype=np.float64)
+        assert np.all(w > 0), "causal-probability scores must be positive"
+        r = float((np.abs(g - w) / w).max())
+        assert r <= rel, f"a: max relative err {r:.3g} > {rel}"
+    return e
+
+
 def check_floats(gpu: dict, ref: dict, tol=TOL, mass=True):
-    errs = {"a": assert_close("a", gpu["a"], ref["a"], tol)}
+    causal = ref.get("score_mode", orc.SCORE_CAUSAL_PROB) == orc.SCORE_CAUSAL_PROB
+    errs = {"a": check_a(gpu["a"], ref["a"], causal, tol)}
     if mass and gpu.get("mass") is not None:
         m = gpu["mass"]
         errs["mass"] = assert_close("mass", m[..., :3], ref["mass"], tol)
