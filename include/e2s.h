@@ -245,11 +245,12 @@ e2s_status e2s_fuse_select(const e2s_layout* layout, const e2s_params* params,
  * running inside a host framework whose memory pool owns the whole device
  * heap, plug-ins reached through a foreign-function interface that has no
  * allocator, or real-time loops where cudaMalloc is not allowed.  This entry
- * point takes the same inputs and outputs as e2s_fuse and computes the same
- * results with a two-kernel formulation (a statistics kernel, then one thread
- * per token) whose scratch -- the per-(image, layer, head) normalisation
- * statistics -- lives in a static device array inside the library, so it
- * allocates nothing and needs no workspace.
+ * point takes the same inputs and outputs as e2s_fuse, and its results equal
+ * e2s_fuse's up to the rounding order of the normalisation sums.  It uses a
+ * two-kernel formulation (a statistics kernel, then one thread per token)
+ * whose scratch -- the per-(image, layer, head) normalisation statistics --
+ * lives in a static device array inside the library, so it allocates
+ * nothing and needs no workspace.
  *   - Capacity: B * L * H <= 8192; larger batches return E2S_ERR_WORKSPACE
  *     before anything is launched.  The array (about 64 KiB) is held by every
  *     GPU that loads the library until the process exits.
@@ -262,7 +263,9 @@ e2s_status e2s_fuse_select(const e2s_layout* layout, const e2s_params* params,
  *     reads, so the contents left by an earlier call do no harm.
  *   - Device-side layout errors are not reported (there is no status word to
  *     read back); use e2s_fuse with a workspace and e2s_read_status to
- *     diagnose them. */
+ *     diagnose them.  The tokens of an image whose device layout arrays
+ *     disagree get defined placeholder outputs: every layer mass and the
+ *     fused mass (0, 0, 1, 0) and q = 0. */
 e2s_status e2s_fuse_noalloc(const e2s_layout* layout, const e2s_params* params,
                             const float* a, const int32_t* cand, const float* prior,
                             float* mass_out, float* fused_out, float* q_out, void* stream);
@@ -313,6 +316,21 @@ e2s_status e2s_clear_status(void* ws, void* stream);
 
 /* Human-readable name of a status value (static string). */
 const char* e2s_status_string(e2s_status s);
+
+/* Self-test of the bounded device waits (no counterpart in the paper).
+ * Every mbarrier wait in this library's kernels gives up after a wall-clock
+ * limit, records E2S_ERR_TIMEOUT in the status word and lets the kernel
+ * return, so a lost arrival is reported instead of hanging the GPU.  This
+ * call launches one thread that initialises a barrier expecting two
+ * arrivals, arrives once (twice when `complete` is non-zero) and waits on it
+ * with that same bounded wait, nothing else in flight.
+ *   complete  0: the phase never completes; after limit_ns the wait gives up
+ *             and E2S_ERR_TIMEOUT is OR-ed into the status word.
+ *             1: the phase completes and nothing is recorded.
+ *   limit_ns  HOST value, 1e6 .. 2e9 (1 ms .. 2 s), else E2S_ERR_INVALID_ARG.
+ *   ws        256-byte aligned workspace; only its status word is used.
+ * Read the outcome with e2s_read_status. */
+e2s_status e2s_selftest_bounded_wait(int32_t complete, int64_t limit_ns, void* ws, void* stream);
 
 /* Library ABI version (major * 100 + minor). */
 int32_t e2s_version(void);

@@ -416,6 +416,6 @@ const char* e2s_status_string(e2s_status s) {
   return "E2S_ERR_UNKNOWN";
 }
 
-int32_t e2s_version(void) { return 101; }
+int32_t e2s_version(void) { return 102; }
 
 }  // extern "C"

@@ -21,6 +21,12 @@ namespace {
 constexpr int kStatsThreads = 256;
 constexpr int kTokenThreads = 128;
 
+// Whether image b's device layout arrays agree with each other and with the
+// host totals.  Both kernels take the same decision for the same image.
+__device__ __forceinline__ bool image_layout_ok(const LayoutArgs& la, int b, int NV, int v0) {
+  return NV >= 0 && v0 >= 0 && v0 + NV <= la.sum_vis && __ldg(la.vis_off + b + 1) - v0 == NV;
+}
+
 __global__ void __launch_bounds__(kStatsThreads)
     fuse_stats_kernel(const LayoutArgs la, int softmax, const float* __restrict__ a,
                       float2* __restrict__ stats, uint32_t* status) {
@@ -32,7 +38,7 @@ __global__ void __launch_bounds__(kStatsThreads)
   const int l = (unit / la.H) % la.L;
   const int b = unit / (la.H * la.L);
   const int NV = __ldg(la.n_vis + b), v0 = __ldg(la.vis_off + b);
-  if (NV < 0 || v0 < 0 || v0 + NV > la.sum_vis || __ldg(la.vis_off + b + 1) - v0 != NV) {
+  if (!image_layout_ok(la, b, NV, v0)) {
     if (threadIdx.x == 0) {
       E2S_DEV_FLAG(status, E2S_ERR_SHAPE);
       stats[unit] = make_float2(0.f, 0.f);
@@ -83,6 +89,15 @@ __global__ void __launch_bounds__(kTokenThreads)
   const int H = la.H;
   const float inv_h = 1.f / (float)H;
   const size_t plane = (size_t)la.sum_vis;
+  if (!image_layout_ok(la, b, NV, __ldg(la.vis_off + b))) {
+    // The statistics kernel skipped this image (its entries are zero), so
+    // the evidence is undefined: write the vacuous mass, no conflict, q = 0.
+    if (mass_out)
+      for (int l = 0; l < la.L; ++l) mass_out[(size_t)l * plane + gv] = make_float4(0.f, 0.f, 1.f, 0.f);
+    fused_out[gv] = make_float4(0.f, 0.f, 1.f, 0.f);
+    q_out[gv] = 0.f;
+    return;
+  }
 
   float fI = 0.f, fU = 0.f, fT = 1.f, K = 0.f;
   bool have = false;

@@ -93,6 +93,7 @@ _SIGS = {
     "e2s_read_status": (ctypes.c_int, [_vp, _vp]),
     "e2s_clear_status": (ctypes.c_int, [_vp, _vp]),
     "e2s_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "e2s_selftest_bounded_wait": (ctypes.c_int, [_i32, _i64, _vp, _vp]),
     "e2s_version": (ctypes.c_int32, []),
 }
 for _name, (_res, _args) in _SIGS.items():
@@ -215,6 +216,10 @@ def e2s_fuse_select(layout, params_, a, cand, prior, mass_out, fused_out, q_out,
                                _ptr(mass_out), _ptr(fused_out), _ptr(q_out), _ptr(keep_count),
                                _ptr(keep_off), sum_keep, _ptr(keep_idx), _ptr(q_tilde_out),
                                _ptr(ws), ws_bytes, _stream(stream))
+
+
+def e2s_selftest_bounded_wait(complete: int, limit_ns: int, ws, stream=None) -> int:
+    return lib.e2s_selftest_bounded_wait(int(complete), int(limit_ns), _ptr(ws), _stream(stream))
 
 
 def e2s_fuse_noalloc(layout, params_, a, cand, prior, mass_out, fused_out, q_out,

@@ -57,7 +57,7 @@ def test_workspace_size_and_versions():
     # status word, one float4 per (image, layer, head), 64 cell keys + a counter per image
     assert n == 256 + ((1 * 2 * 32 * 16 + 255) // 256) * 256 + ((1 * 129 * 4 + 255) // 256) * 256
     assert e2s.e2s_workspace_size(_layout(e2s, d=64), e2s.params()) == 0
-    assert e2s.e2s_version() == 101
+    assert e2s.e2s_version() == 102
     assert e2s.e2s_status_string(e2s.E2S_ERR_TIMEOUT) == "E2S_ERR_TIMEOUT"
     assert e2s.e2s_status_string(99) == "E2S_ERR_UNKNOWN"
 
@@ -220,3 +220,11 @@ def test_decide_host_validation(case, want):
                         a, None, fused, 0x580000, keep_count, 0x680000, 64, keep_idx, None,
                         ws, wsb, None)
     assert e2s.e2s_status_string(st) == want
+
+
+def test_selftest_bounded_wait_host_validation():
+    e2s = _lib()
+    assert e2s.e2s_selftest_bounded_wait(0, 50_000_000, None) == e2s.E2S_ERR_WORKSPACE
+    assert e2s.e2s_selftest_bounded_wait(0, 50_000_000, 0x1010) == e2s.E2S_ERR_WORKSPACE
+    assert e2s.e2s_selftest_bounded_wait(0, 10, 0x1000) == e2s.E2S_ERR_INVALID_ARG
+    assert e2s.e2s_selftest_bounded_wait(0, 3_000_000_000, 0x1000) == e2s.E2S_ERR_INVALID_ARG

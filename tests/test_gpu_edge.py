@@ -236,3 +236,26 @@ def test_call_sequences_agree(path):
         parity.assert_close(key, g1[key], g2[key], tol=1e-5)
     for b in range(4):
         assert np.array_equal(g1["keep"][b], g2["keep"][b])
+
+
+def test_bounded_wait_reports_timeout_and_context_survives():
+    """A bounded mbarrier wait whose phase never completes gives up after its
+    limit, records E2S_ERR_TIMEOUT and lets the kernel return: the host reads
+    the status and the context still runs a decision afterwards."""
+    import time
+    from paper_2608_23253_gb300 import e2s
+    dev = device()
+    ws = torch.zeros(64, dtype=torch.int32, device=dev)
+    assert ws.data_ptr() % 256 == 0
+    assert e2s.e2s_selftest_bounded_wait(1, 50_000_000, ws) == e2s.E2S_OK
+    assert e2s.e2s_read_status(ws, None) == e2s.E2S_OK
+    t0 = time.perf_counter()
+    assert e2s.e2s_selftest_bounded_wait(0, 50_000_000, ws) == e2s.E2S_OK
+    assert e2s.e2s_read_status(ws, None) == e2s.E2S_ERR_TIMEOUT
+    assert time.perf_counter() - t0 >= 0.05
+    assert e2s.e2s_clear_status(ws, None) == e2s.E2S_OK
+    assert e2s.e2s_read_status(ws, None) == e2s.E2S_OK
+    inp = config_inputs(0, None, None)
+    gpu = run_gpu(inp, "causal")
+    assert gpu["status"] == 0
+    parity.check_floats(gpu, run_oracle(inp, "causal"))
