@@ -27,7 +27,9 @@ LLaVA-1.5-7B and Qwen2-VL-7B settings of Sec. 4.1 and Table 5):
 """
 from __future__ import annotations
 
+import concurrent.futures as cf
 import dataclasses
+import os
 from typing import List, Optional, Sequence
 
 import numpy as np
@@ -36,11 +38,23 @@ D_HEAD = 128
 SIGMA = D_HEAD ** -0.25
 
 
-def bf16_bits(x: np.ndarray) -> np.ndarray:
-    """Round float32 values to bf16 (nearest-even) and return the bit patterns."""
-    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
-    rounded = u + (np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1)))
-    return (rounded >> np.uint32(16)).astype(np.uint16)
+def bf16_bits(x: np.ndarray, chunk: int = 1 << 20) -> np.ndarray:
+    """Round float32 values to bf16 (nearest-even) and return the bit patterns:
+    (u + 0x7FFF + ((u >> 16) & 1)) >> 16 on the float's bits, in place over
+    cache-sized chunks."""
+    u = np.ascontiguousarray(x, dtype=np.float32).reshape(-1).view(np.uint32)
+    out = np.empty(u.shape, dtype=np.uint16)
+    tmp = np.empty(min(chunk, max(u.size, 1)), dtype=np.uint32)
+    for s in range(0, u.size, chunk):
+        e = min(s + chunk, u.size)
+        r = tmp[:e - s]
+        np.right_shift(u[s:e], 16, out=r)
+        r &= np.uint32(1)
+        r += np.uint32(0x7FFF)
+        r += u[s:e]
+        r >>= np.uint32(16)
+        out[s:e] = r
+    return out.reshape(np.shape(x))
 
 
 def bf16_to_f32(bits: np.ndarray) -> np.ndarray:
@@ -220,15 +234,15 @@ def make_inputs(spec: Spec, *, with_payload: bool = True) -> Inputs:
     payload = with_payload and spec.hidden > 0
     v = np.empty((L, sum_T, Hkv, d), dtype=np.uint16) if payload else None
     hid = np.empty((sum_T, spec.hidden), dtype=np.uint16) if payload else None
-    salient = []
     amp = SIGMA * np.sqrt(d)
-    for b, im in enumerate(spec.images):
+
+    def draw_image(b: int) -> np.ndarray:
+        im = spec.images[b]
         rng = np.random.Generator(np.random.PCG64(1000 * spec.cfg_id + b))
         # V and the hidden states come from a stream of their own, so Q and K
         # are the same with or without the payload
         prng = np.random.Generator(np.random.PCG64(1000 * spec.cfg_id + b + (1 << 40)))
         sal = _salient_positions(rng, im.grid_h, im.grid_w, im.n_salient, im.blobs)
-        salient.append(sal)
         t0, t1 = int(tok_off[b]), int(tok_off[b + 1])
         x0, x1 = int(text_off[b]), int(text_off[b + 1])
         for l in range(L):
@@ -246,6 +260,14 @@ def make_inputs(spec: Spec, *, with_payload: bool = True) -> Inputs:
                 v[l, t0:t1] = bf16_bits(prng.standard_normal((t1 - t0, Hkv, d), dtype=np.float32))
         if payload:
             hid[t0:t1] = bf16_bits(prng.standard_normal((t1 - t0, spec.hidden), dtype=np.float32))
+        return sal
+
+    # Images draw from streams of their own and write disjoint rows, so they
+    # run on a thread pool (numpy releases the GIL while it fills the arrays);
+    # the values do not depend on the number of threads.
+    workers = max(1, min(B, os.cpu_count() or 1, 16))
+    with cf.ThreadPoolExecutor(max_workers=workers) as ex:
+        salient = list(ex.map(draw_image, range(B)))
     return Inputs(spec, n_sys, n_vis, n_text, grid_h, grid_w, tok_off, vis_off, text_off,
                   keep, keep_off, q, k, v, hid, salient)
 

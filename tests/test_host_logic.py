@@ -136,3 +136,13 @@ def test_bench_attention_lse_matches_oracle():
     want = orc.text_row_lse(inp.q_text, inp.k, inp.n_sys, inp.n_vis, inp.n_text, H_kv=2)
     assert got.shape == want.shape
     assert np.abs(got - want).max() < 1e-4
+
+
+def test_bench_ablation_flags_parse_to_the_header_values():
+    """bench --flags: Table 2's A1..A5 names map to the E2S_* flag bits."""
+    import bench
+    assert bench.parse_flags("") == 0
+    assert bench.parse_flags("A1") == 16 and bench.parse_flags("a2") == 1
+    assert bench.parse_flags("A3,A4") == 2 | 4 and bench.parse_flags("A5") == 8
+    assert bench.parse_flags("0x6") == 6
+    assert {v[1] for v in bench.ABLATIONS.values()} == {1, 2, 4, 8, 16}
