@@ -123,7 +123,7 @@ __host__ __device__ inline SPlan stream_plan(int stages) {
   s.q = 0;                                              // [2 halves][128 rows][128 B]
   s.k = (uint32_t)kTileBytes;                           // [stages][tile]
   s.bars = s.k + (uint32_t)stages * kTileBytes;         // mbarriers, see the kernel
-  s.slot = s.bars + 8u * (uint32_t)(2 + 2 * kMaxStages + 4 + kMaxBatch + 1);
+  s.slot = s.bars + 8u * (uint32_t)(2 + 2 * kMaxStages + 4 + kMaxBatch + 2);
   s.ms = (s.slot + 16u + 15u) & ~15u;                   // [4][128] float2 (max, sum)
   s.lse = s.ms + 4u * kRows * 8u;                       // [128] float -lse per text row
   s.cps = s.lse + kRows * 4u;                           // [2][8 chunks][128 keys] partials
@@ -221,6 +221,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* a_empty = a_full + 2;          // [2] accumulator buffer read
   uint64_t* b_full = a_empty + 2;          // [kMaxBatch] batch sweep-2 accumulator ready
   uint64_t* b_done = b_full + kMaxBatch;   // batch sweep 2 read: TMEM free again
+  uint64_t* s1_done = b_done + 1;          // a batch unit's sweep-1 accumulators all read
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + plan.slot);
   float2* ms = reinterpret_cast<float2*>(smem + plan.ms);
   float* nlse = reinterpret_cast<float*>(smem + plan.lse);   // -lse per text row
@@ -248,6 +249,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < kMaxBatch; ++i) ptx::mbar_init(b_full + i, 1);
     ptx::mbar_init(b_done, kEpiWarps);
+    ptx::mbar_init(s1_done, kEpiWarps);
     ptx::fence_barrier_init();
     ptx::fence_proxy_async_smem();
     ptx::prefetch_tensormap(&tmQ);
@@ -379,12 +381,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (g.batch && mid == 0) {
           // every sweep-1 accumulator read: the sweep-2 accumulators of all
-          // visual tiles go side by side into TMEM columns j * n2c
-          for (int k = 1; k <= 2; ++k) {
-            const int tp = tc - k;
-            if (tp >= 0 && !ptx::mbar_wait(a_empty + (tp & 1), (tp / 2) & 1, limit, p.status))
-              limit = kWaitNsAfterFault;
-          }
+          // visual tiles go side by side into TMEM columns j * n2c.  The wait is
+          // on a barrier that completes once per batch unit: a parity wait on
+          // the other issuer's a_empty buffer could see a phase two behind
+          // (that issuer not yet past its previous tile) and pass at once.
+          if (!ptx::mbar_wait(s1_done, bu & 1, limit, p.status)) limit = kWaitNsAfterFault;
           ptx::tc_fence_after();
           for (int j = 0; j < kMaxBatch; ++j) {
             if (j < g.n2) {
@@ -470,6 +471,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(a_empty + buf);
       }
+      // a batch unit's sweep-2 MMAs overwrite both accumulator buffers: they
+      // wait until every warp has read its last sweep-1 tile
+      if (g.batch && lane == 0) ptx::mbar_arrive(s1_done);
       // ---- merge the four column groups: lse per row (log2 domain), published
       // per text row for sweep 2 (or taken from the caller's attention pass)
       if (causal && p.lse_in != nullptr) {
