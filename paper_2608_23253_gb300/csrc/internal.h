@@ -77,6 +77,14 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
                                 const void* k, int64_t k_stride, float* a_out, float4* stats,
                                 uint32_t* counters, uint32_t* status, cudaStream_t st,
                                 const float* lse_in = nullptr);
+// Cluster-per-unit score kernel for small batches (key tiles split over the
+// cluster's CTAs): its cluster size and tiles per CTA, or false when it does
+// not take the launch.  lse_in as for launch_score_stream.
+bool score_split_plan(const LayoutArgs& la, int mode, bool lse, int* cluster, int* tpc);
+cudaError_t launch_score_split(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
+                               const void* k, int64_t k_stride, float* a_out, float4* stats,
+                               uint32_t* counters, uint32_t* status, cudaStream_t st,
+                               const float* lse_in, int cluster, int tpc);
 // Persistent single-CTA-per-unit score kernel and its applicability tests.
 bool score_unit_fits(const LayoutArgs& la, int mode);
 bool score_unit_single_group(const LayoutArgs& la, int mode);

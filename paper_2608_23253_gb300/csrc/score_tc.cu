@@ -504,11 +504,17 @@ cudaError_t launch_score_tc(const LayoutArgs& la, int mode, const void* q, int64
                             uint32_t* counters, uint32_t* status, cudaStream_t st,
                             int* unsupported) {
   *unsupported = 0;
-  // kernel choice (measured): the persistent single-CTA kernel when every
+  // kernel choice (measured): the cluster-per-unit kernel when every unit's
+  // key tiles spread over at most two CTAs per SM in one wave (batch 1); the
+  // persistent single-CTA kernel when every
   // unit's logits fit TMEM in one column group (short sequences, e.g. one
   // LLaVA image); the streaming kernel for longer sequences, GQA and batched
   // ragged text (up to 128 text rows); the column-group kernel above 128 text
   // rows while the K tiles fit shared memory; the cluster kernel otherwise
+  int split_c = 0, split_t = 0;
+  if (score_split_plan(la, mode, false, &split_c, &split_t))
+    return launch_score_split(la, mode, q, q_stride, k, k_stride, a_out, stats, counters, status,
+                              st, nullptr, split_c, split_t);
   const bool unit = score_unit_fits(la, mode);
   if (unit && score_unit_single_group(la, mode))
     return launch_score_unit(la, mode, q, q_stride, k, k_stride, a_out, stats, counters, status,

@@ -200,16 +200,22 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
 }
 
 // 32 lanes x 16 columns of 32-bit TMEM words: thread i gets lane (base + i).
+// tcgen05.ld writes its registers asynchronously; they are valid only after
+// tcgen05.wait::ld.  Both sit in one asm statement, so the registers are
+// outputs of the wait and no use of them can be scheduled before it (with a
+// separate wait statement the compiler sees no dependency between the wait
+// and the registers and may move arithmetic on them ahead of it).
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   uint32_t r[16];
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
       : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
         "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
         "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+      : "r"(taddr)
+      : "memory");
 #pragma unroll
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
@@ -281,6 +287,23 @@ __device__ __forceinline__ float ld_dsmem_f32(const void* local_ptr, uint32_t ra
   return v;
 }
 
+// Arrive on the cluster barrier without ordering earlier memory operations
+// (a start-of-kernel rendezvous: every CTA of the cluster is running).
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory");
+}
+// Store a float2 / float4 into the shared memory of CTA `rank` of this cluster.
+__device__ __forceinline__ void st_dsmem_f2(void* local_ptr, uint32_t rank, float2 v) {
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(dsmem_addr(local_ptr, rank)),
+               "f"(v.x), "f"(v.y)
+               : "memory");
+}
+__device__ __forceinline__ void st_dsmem_f4(void* local_ptr, uint32_t rank, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(
+                   dsmem_addr(local_ptr, rank)),
+               "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+               : "memory");
+}
 // Store a float into the shared memory of CTA `rank` of this cluster.
 __device__ __forceinline__ void st_dsmem_f32(void* local_ptr, uint32_t rank, float v) {
   asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(dsmem_addr(local_ptr, rank)), "f"(v)

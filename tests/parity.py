@@ -44,7 +44,14 @@ def max_err(got, want) -> float:
 
 def assert_close(name, got, want, tol=TOL):
     e = max_err(got, want)
-    assert e <= tol, f"{name}: max abs err {e:.3g} > {tol}"
+    if e > tol:
+        g = np.asarray(got, dtype=np.float64)
+        w = np.asarray(want, dtype=np.float64)
+        d = np.abs(g - w)
+        at = np.unravel_index(int(np.argmax(d)), d.shape)
+        n_bad = int((d > tol).sum())
+        raise AssertionError(f"{name}: max abs err {e:.3g} > {tol} at {tuple(int(i) for i in at)} "
+                             f"(got {g[at]:.6g}, want {w[at]:.6g}; {n_bad} of {d.size} beyond)")
     return e
 
 

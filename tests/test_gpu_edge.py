@@ -259,3 +259,54 @@ def test_bounded_wait_reports_timeout_and_context_survives():
     gpu = run_gpu(inp, "causal")
     assert gpu["status"] == 0
     parity.check_floats(gpu, run_oracle(inp, "causal"))
+
+
+@pytest.mark.parametrize("mode", ["causal", "eq1"])
+def test_two_llava_images_persistent_unit_kernel(mode):
+    """Two LLaVA-1.5-7B-shaped images (35 + 24x24 + 64 tokens, 3 layers, 32
+    heads): 192 units are more than one wave of the cluster-per-unit kernel,
+    so the persistent one-CTA-per-unit score kernel takes them."""
+    ims = [ImageSpec(35, 24, 24, 64, 40, 3, 64), ImageSpec(35, 24, 24, 64, 40, 3, 128)]
+    spec = synth.custom_spec("llava-b2", ims, L=3, H=32, H_kv=32)
+    inp = synth.make_inputs(spec, with_payload=False)
+    gpu = run_gpu(inp, mode)
+    assert gpu["status"] == 0
+    ref = run_oracle(inp, mode)
+    parity.check_floats(gpu, ref)
+    parity.check_selection(gpu["keep"], gpu["q_tilde"], ref["q"], inp.n_vis, inp.grid_h,
+                           inp.grid_w, inp.keep, 0.1, 4)
+
+
+@pytest.mark.parametrize("cfg,batch,reps", [(2, 6, 400), (2, None, 60), (1, None, 200)],
+                         ids=["llava-ragged-b6", "llava-ragged-b32", "llava-b1"])
+def test_prune_repeats_bit_identical(cfg, batch, reps):
+    """The whole step (e2s_prune: score, decision and compaction overlapping
+    through programmatic dependent launch) repeated back to back gives the
+    same scores and keep sets bit for bit every time.  The decision and
+    compaction kernels share the SMs with the score kernel, so their timing
+    varies from call to call; a missing wait inside the score kernel shows
+    up here as a call whose scores differ."""
+    from paper_2608_23253_gb300 import e2s
+    from paper_2608_23253_gb300.decision import Batch, Decision, bf16_tensor
+    dev = device()
+    inp = config_inputs(cfg, batch, None, True)
+    dec = Decision(Batch.from_inputs(inp, device=dev), inp.keep, e2s.params())
+    L = inp.spec.L
+    host = [inp.hidden] + [inp.k[l].reshape(inp.k.shape[1], -1) for l in range(L)] + \
+           [inp.v[l].reshape(inp.v.shape[1], -1) for l in range(L)]
+    src = [bf16_tensor(x, dev) for x in host]
+    dst = [torch.empty((dec.out_rows(), t.shape[1]), dtype=t.dtype, device=dev) for t in src]
+    pos = torch.empty(dec.out_rows(), dtype=torch.int32, device=dev)
+    q, k = bf16_tensor(inp.q_text, dev), bf16_tensor(inp.k, dev)
+    first_a = first_keep = None
+    for it in range(reps):
+        dec.a.fill_(float("nan"))
+        dec.prune(q, k, src, dst, pos)
+        a, keep = dec.a.clone(), dec.keep_idx.clone()
+        if first_a is None:
+            first_a, first_keep = a, keep
+            continue
+        same = torch.equal(a.view(torch.int32), first_a.view(torch.int32))
+        assert same and torch.equal(keep, first_keep), f"call {it} differs from the first"
+    torch.cuda.synchronize()
+    assert dec.status() == 0
