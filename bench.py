@@ -70,10 +70,10 @@ WORKLOADS = {
 # sha256 (first 16 hex) of the kernel's sources (its .cu and the device headers
 # it includes) when it was captured; sources that have changed since report
 # null traffic.
-KERNEL_SOURCES = ("score_unit.cu", "sm100_ptx.cuh", "device_common.cuh")
+KERNEL_SOURCES = ("score_split.cu", "sm100_ptx.cuh", "device_common.cuh")
 NCU_TRAFFIC = {
-    "cfg1": {"stage": "score", "kernel": "score_unit_kernel", "src": KERNEL_SOURCES,
-             "sha": "0f6e171e130388e8", "bytes": 18230000},
+    "cfg1": {"stage": "score", "kernel": "score_split_kernel", "src": KERNEL_SOURCES,
+             "sha": "70b211816da11f00", "bytes": 18226688},
 }
 
 
@@ -88,14 +88,14 @@ ABLATIONS = {"A1": ("vanilla: q = mean attention, no novelty", 16),
 # (profiles/score_*_kernel_*.md), with the source hash they were taken on.
 STREAM_SOURCES = ("score_stream.cu", "sm100_ptx.cuh", "device_common.cuh")
 NCU_TENSOR_PIPE = {
-    "cfg1": {"kernel": "score_unit_kernel", "src": KERNEL_SOURCES, "sha": "0f6e171e130388e8",
-             "pct": 6.36, "profile": "profiles/score_unit_kernel_llava_b1.md"},
-    "cfg2": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "d6da10b297b675ce",
-             "pct": 24.63, "profile": "profiles/score_stream_kernel_llava_b32.md"},
-    "cfg3": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "d6da10b297b675ce",
-             "pct": 33.47, "profile": "profiles/score_stream_kernel_qwen2vl_b16.md"},
-    "cfg4": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "d6da10b297b675ce",
-             "pct": 36.62, "profile": "profiles/score_stream_kernel_highres_b8.md"},
+    "cfg1": {"kernel": "score_split_kernel", "src": KERNEL_SOURCES, "sha": "70b211816da11f00",
+             "pct": 15.71, "profile": "profiles/score_split_kernel_llava_b1.md"},
+    "cfg2": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "a6aa69b8ca205fe5",
+             "pct": 25.19, "profile": "profiles/score_stream_kernel_llava_b32.md"},
+    "cfg3": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "a6aa69b8ca205fe5",
+             "pct": 32.92, "profile": "profiles/score_stream_kernel_qwen2vl_b16.md"},
+    "cfg4": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "a6aa69b8ca205fe5",
+             "pct": 37.55, "profile": "profiles/score_stream_kernel_highres_b8.md"},
 }
 
 
