@@ -6,7 +6,9 @@ Follows the paper step by step, in the order of Algorithm 1:
   Sec. 4.2 Eqs. 12-19       Dempster-Shafer fusion across layers, Bel, Pl, priority q
   Sec. 4.3 Eqs. 20-23       spatial cell representative, indicator b, q~, Top-K
 and the compaction of the retained rows that the shortened sequence implies
-(Sec. 4 opening paragraph; Sec. 5.1.2 pruning settings).
+(Sec. 4 opening paragraph; Sec. 5.1.2 pruning settings).  causal_attention_output
+and attention_layer give the pruning layer's own causal attention (output and
+row normalisers), whose text rows the score reads.
 
 Readings where the paper is silent or ambiguous (each one is listed in the
 design notes as well):
@@ -99,6 +101,21 @@ def causal_row_lse(Q: np.ndarray, K_all: np.ndarray, first_text_pos: int) -> np.
     z = np.where(visible, logits, -np.inf)
     m = z.max(axis=1)
     return m + np.log(np.exp(z - m[:, None]).sum(axis=1))
+
+
+def causal_attention_output(Q_all: np.ndarray, K_all: np.ndarray, V_all: np.ndarray):
+    """Causal self-attention of one head over one image (Sec. 3.1): row p
+    attends to keys 0..p with weights softmax_j(Q_p K_j / sqrt(d)); returns
+    (O [T, d] = P V, lse [T] natural-log normaliser of each row)."""
+    d = Q_all.shape[1]
+    T = K_all.shape[0]
+    logits = Q_all @ K_all.T / np.sqrt(d)      # [T, T]
+    visible = np.arange(T)[None, :] <= np.arange(Q_all.shape[0])[:, None]
+    z = np.where(visible, logits, -np.inf)
+    m = z.max(axis=1)
+    e = np.where(visible, np.exp(z - m[:, None]), 0.0)
+    s = e.sum(axis=1)
+    return (e / s[:, None]) @ V_all, m + np.log(s)
 
 
 def score_causal_prob(Q: np.ndarray, K_all: np.ndarray, S: int, N_V: int) -> np.ndarray:
@@ -308,6 +325,29 @@ def text_row_lse(q_text, k, n_sys, n_vis, n_text, *, H_kv: int) -> np.ndarray:
         t0 += T
         x0 += N_T
     return out
+
+
+def attention_layer(q_all, k, v, n_sys, n_vis, n_text, *, H_kv: int):
+    """Causal attention of every image, layer and query head of a packed batch:
+    q_all uint16 [L, sum T, H, d], k / v uint16 [L, sum T, H_kv, d] (bf16 bits).
+    Returns O [L, sum T, H, d] and lse [L, H, sum T] (float64); query head h
+    reads kv head floor(h / (H / H_kv))."""
+    L, sum_T, H, d = q_all.shape
+    group = H // H_kv
+    O = np.zeros((L, sum_T, H, d))
+    lse = np.zeros((L, H, sum_T))
+    t0 = 0
+    for b in range(len(n_sys)):
+        T = int(n_sys[b]) + int(n_vis[b]) + int(n_text[b])
+        for l in range(L):
+            for h in range(H):
+                o, ls = causal_attention_output(widen_bf16(q_all[l, t0:t0 + T, h]),
+                                                widen_bf16(k[l, t0:t0 + T, h // group]),
+                                                widen_bf16(v[l, t0:t0 + T, h // group]))
+                O[l, t0:t0 + T, h] = o
+                lse[l, h, t0:t0 + T] = ls
+        t0 += T
+    return O, lse
 
 
 def image_evidence(a: np.ndarray, params: Params) -> Dict[str, np.ndarray]:

@@ -96,3 +96,19 @@ def test_lse_prefix_off_by_one_is_caught():
     bad = np.array([logsumexp(logits[t, :4 + t]) for t in range(3)])
     assert np.allclose(orc.causal_row_lse(Q, K, 4), want, atol=1e-12)
     assert not np.allclose(bad, want, atol=1e-6)
+
+
+def test_attention_mask_including_the_next_key_is_caught():
+    """An attention mask one key too wide ('<= p + 1') fails the identity-value pin."""
+    from scipy.special import softmax
+    r = np.random.default_rng(43)
+    T, d = 6, 4
+    Q, K = r.normal(size=(T, d)), r.normal(size=(T, d))
+    logits = Q @ K.T / 2.0
+    vis = np.arange(T)[None, :] <= np.arange(T)[:, None] + 1
+    z = np.where(vis, logits, -np.inf)
+    bad = np.exp(z - z.max(axis=1, keepdims=True))
+    bad = bad / bad.sum(axis=1, keepdims=True)
+    good, _ = orc.causal_attention_output(Q, K, np.eye(T))
+    assert np.allclose(good[2, :3], softmax(logits[2, :3]))
+    assert not np.allclose(bad[2, :3], softmax(logits[2, :3]))

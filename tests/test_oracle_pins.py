@@ -405,3 +405,48 @@ def test_causal_row_lse_reconstructs_attention_rows():
         assert np.all(P[t, n:] == 0)
     one = orc.causal_row_lse(Q[:1], K, 0)
     assert abs(one[0] - logits[0, 0]) < 1e-14
+
+
+# ------------------------------------------------------ the layer's attention
+def test_attention_output_with_identity_values_is_the_softmax_rows():
+    """V = identity: O = P, each row a textbook softmax of the visible logits
+    (scipy), zero beyond the row's own position; lse is scipy's logsumexp."""
+    from scipy.special import logsumexp
+    r = _rng(40)
+    T, d = 9, 8
+    Q, K = r.normal(size=(T, d)), r.normal(size=(T, d))
+    O, lse = orc.causal_attention_output(Q, K, np.eye(T))
+    logits = Q @ K.T / math.sqrt(d)
+    for p in range(T):
+        np.testing.assert_allclose(O[p, :p + 1], sp_softmax(logits[p, :p + 1]), atol=1e-14)
+        assert np.all(O[p, p + 1:] == 0)
+        assert abs(lse[p] - logsumexp(logits[p, :p + 1])) < 1e-12
+
+
+def test_attention_output_special_cases():
+    r = _rng(41)
+    T, d = 7, 4
+    Q, K, V = r.normal(size=(T, d)), r.normal(size=(T, d)), r.normal(size=(T, 5))
+    O, _ = orc.causal_attention_output(Q, K, V)
+    np.testing.assert_allclose(O[0], V[0], atol=1e-15)             # the first row sees one key
+    O2, _ = orc.causal_attention_output(Q, K, np.tile(V[3], (T, 1)))
+    np.testing.assert_allclose(O2, np.tile(V[3], (T, 1)), atol=1e-14)   # equal values: O = v
+    # brute force with math.exp for the last row
+    lg = [sum(Q[T - 1, i] * K[j, i] for i in range(d)) / math.sqrt(d) for j in range(T)]
+    w = [math.exp(x - max(lg)) for x in lg]
+    want = [sum(w[j] * V[j, c] for j in range(T)) / sum(w) for c in range(5)]
+    np.testing.assert_allclose(O[T - 1], want, atol=1e-13)
+
+
+def test_attention_text_rows_give_the_score_and_row_lse():
+    """The text rows of the layer's attention carry the decision's inputs:
+    their lse equals causal_row_lse, and the mean of their probabilities on
+    the visual keys (recovered as O with identity values) is a."""
+    r = _rng(42)
+    S, NV, NT, d = 3, 6, 4, 8
+    T = S + NV + NT
+    Q, K = r.normal(size=(T, d)), r.normal(size=(T, d))
+    O, lse = orc.causal_attention_output(Q, K, np.eye(T))
+    np.testing.assert_allclose(lse[S + NV:], orc.causal_row_lse(Q[S + NV:], K, S + NV), atol=1e-12)
+    np.testing.assert_allclose(O[S + NV:, S:S + NV].mean(axis=0),
+                               orc.score_causal_prob(Q[S + NV:], K, S, NV), atol=1e-15)
