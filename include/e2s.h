@@ -146,6 +146,52 @@ e2s_status e2s_score_lse(const e2s_layout* layout, const e2s_params* params,
                          const void* k, int64_t k_row_stride, const float* lse_text,
                          float* a_out, void* ws, size_t ws_bytes, void* stream);
 
+/* The pruning layer's own causal self-attention, with the decision's score
+ * as a by-product (Sec. 3.1; Sec. 6 names lower-overhead evidence caching as
+ * future work, and reading the score off the layer's attention pass is this
+ * library's reading of it).  Every row attends to the keys of its own image
+ * at positions up to its own (causal mask per image, images packed as in the
+ * layout); query head h uses key/value head h / (H / H_kv).
+ *   q        bf16 [L][sum_T] rows of (H x d): the queries of EVERY row (not
+ *            only the text rows), row stride q_row_stride elements.
+ *   k, v     bf16 [L][sum_T] rows of (H_kv x d), strides k_/v_row_stride.
+ *   o_out    bf16 [L][sum_T] rows of (H x d), stride o_row_stride: the
+ *            attention output softmax(Q K^T / sqrt(d)) V of every row.
+ *   lse_out  nullable fp32 [L][H][sum_T]: natural-log normaliser of every row
+ *            (the value e2s_score_lse takes for the text rows).
+ *   a_out    nullable fp32 [L][H][sum_vis]: the CAUSAL_PROB score of
+ *            e2s_score, computed from the final normalisers of the text rows
+ *            inside the same launch (no other pass reads K for it); the Eq. 8
+ *            statistics go to the workspace and the decision scratch is
+ *            zeroed, as e2s_score does, so e2s_fuse / e2s_fuse_select /
+ *            e2s_select may follow.  Requires max_text <= 128
+ *            (E2S_ERR_UNSUPPORTED otherwise).
+ * Pointers 16-byte aligned (lse_out, a_out 4), strides multiples of 8 and at
+ * least H*d (q, o) or H_kv*d (k, v).  P is rounded to bf16 before P V, as in
+ * flash-attention forwards, so O carries bf16 rounding of the weights; lse
+ * and a are computed from the fp32 logits. */
+e2s_status e2s_attention(const e2s_layout* layout, const void* q, int64_t q_row_stride,
+                         const void* k, int64_t k_row_stride, const void* v, int64_t v_row_stride,
+                         void* o_out, int64_t o_row_stride, float* lse_out, float* a_out,
+                         void* ws, size_t ws_bytes, void* stream);
+
+
+/* The whole pruning decision from the pruning layer's own attention pass, in
+ * two launches: e2s_attention with a_out (the layer's O and lse, the score a
+ * and its Eq. 8 statistics), then the evidence, fusion and selection of
+ * e2s_decide from them -- no pass of its own over K.  Arguments are those of
+ * e2s_attention and e2s_decide; a_out is required and params->score_mode must
+ * be E2S_SCORE_CAUSAL_PROB (the attention pass defines that score).  Results
+ * equal e2s_decide's up to the rounding order of the score's sums. */
+e2s_status e2s_decide_attn(const e2s_layout* layout, const e2s_params* params, const void* q,
+                           int64_t q_row_stride, const void* k, int64_t k_row_stride,
+                           const void* v, int64_t v_row_stride, void* o_out, int64_t o_row_stride,
+                           float* lse_out, const int32_t* cand, const float* prior, float* a_out,
+                           float* mass_out, float* fused_out, float* q_out,
+                           const int32_t* keep_count, const int32_t* keep_off, int32_t sum_keep,
+                           int32_t* keep_idx, float* q_tilde_out, void* ws, size_t ws_bytes,
+                           void* stream);
+
 /* The whole pruning decision of one step in two launches: e2s_score, then
  * evidence, fusion and selection (Sec. 3.1 and 4.1-4.3, Eqs. 1 and 8-23).
  * Arguments have the meaning they have in e2s_score, e2s_fuse and e2s_select;

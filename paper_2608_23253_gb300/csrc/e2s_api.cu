@@ -246,6 +246,55 @@ e2s_status e2s_score_lse(const e2s_layout* layout, const e2s_params* params, con
                    static_cast<cudaStream_t>(stream), lse_text);
 }
 
+e2s_status e2s_attention(const e2s_layout* layout, const void* q, int64_t q_row_stride,
+                         const void* k, int64_t k_row_stride, const void* v,
+                         int64_t v_row_stride, void* o_out, int64_t o_row_stride, float* lse_out,
+                         float* a_out, void* ws, size_t ws_bytes, void* stream) {
+  E2S_TRY(check_layout(layout));
+  E2S_TRY(check_ws(layout, ws, ws_bytes));
+  if (!q || !k || !v || !o_out) return E2S_ERR_INVALID_ARG;
+  const int64_t hd = (int64_t)layout->H * layout->d, kvd = (int64_t)layout->H_kv * layout->d;
+  if (q_row_stride < hd || o_row_stride < hd || k_row_stride < kvd || v_row_stride < kvd)
+    return E2S_ERR_SHAPE;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o_out) ||
+      (q_row_stride % 8) || (k_row_stride % 8) || (v_row_stride % 8) || (o_row_stride % 8) ||
+      (reinterpret_cast<uintptr_t>(lse_out) & 3u) || (reinterpret_cast<uintptr_t>(a_out) & 3u))
+    return E2S_ERR_ALIGNMENT;
+  if (a_out != nullptr && layout->max_text > 128) return E2S_ERR_UNSUPPORTED;
+  return from_cuda(launch_attention(layout_args(layout), q, q_row_stride, k, k_row_stride, v,
+                                    v_row_stride, o_out, o_row_stride, lse_out, a_out,
+                                    stats_ptr(ws), a_out ? decide_scratch_ptr(ws, layout) : nullptr,
+                                    status_word(ws), static_cast<cudaStream_t>(stream)));
+}
+
+e2s_status e2s_decide_attn(const e2s_layout* layout, const e2s_params* params, const void* q,
+                           int64_t q_row_stride, const void* k, int64_t k_row_stride,
+                           const void* v, int64_t v_row_stride, void* o_out, int64_t o_row_stride,
+                           float* lse_out, const int32_t* cand, const float* prior, float* a_out,
+                           float* mass_out, float* fused_out, float* q_out,
+                           const int32_t* keep_count, const int32_t* keep_off, int32_t sum_keep,
+                           int32_t* keep_idx, float* q_tilde_out, void* ws, size_t ws_bytes,
+                           void* stream) {
+  E2S_TRY(check_params(params));
+  if (params->score_mode != E2S_SCORE_CAUSAL_PROB) return E2S_ERR_UNSUPPORTED;
+  if (!a_out && layout && layout->sum_vis > 0) return E2S_ERR_INVALID_ARG;
+  if (layout && layout->sum_vis > 0 && (!fused_out || !q_out)) return E2S_ERR_INVALID_ARG;
+  if (!keep_count || !keep_off || sum_keep < 0) return E2S_ERR_INVALID_ARG;
+  if (sum_keep > 0 && !keep_idx) return E2S_ERR_INVALID_ARG;
+  if (!aligned16(prior) || !aligned16(mass_out) || !aligned16(fused_out)) return E2S_ERR_ALIGNMENT;
+  E2S_TRY(e2s_attention(layout, q, q_row_stride, k, k_row_stride, v, v_row_stride, o_out,
+                        o_row_stride, lse_out, a_out, ws, ws_bytes, stream));
+  if (!decide_fits(layout_args(layout))) return E2S_ERR_UNSUPPORTED;
+  int unsupported = 0;
+  const cudaError_t e = launch_decide(
+      layout_args(layout), norm_is_softmax(params), params->flags, params->lambda, params->G,
+      a_out, stats_ptr(ws), prior, cand, mass_out, fused_out, q_out, q_tilde_out, keep_count,
+      keep_off, sum_keep, keep_idx, decide_scratch_ptr(ws, layout), status_word(ws),
+      static_cast<cudaStream_t>(stream), &unsupported);
+  if (unsupported) return E2S_ERR_UNSUPPORTED;
+  return from_cuda(e);
+}
+
 e2s_status e2s_decide_lse(const e2s_layout* layout, const e2s_params* params,
                           const void* q_text, int64_t q_row_stride, const void* k,
                           int64_t k_row_stride, const float* lse_text, const int32_t* cand,
@@ -422,6 +471,6 @@ const char* e2s_status_string(e2s_status s) {
   return "E2S_ERR_UNKNOWN";
 }
 
-int32_t e2s_version(void) { return 102; }
+int32_t e2s_version(void) { return 103; }
 
 }  // extern "C"

@@ -85,6 +85,12 @@ cudaError_t launch_score_split(const LayoutArgs& la, int mode, const void* q, in
                                const void* k, int64_t k_stride, float* a_out, float4* stats,
                                uint32_t* counters, uint32_t* status, cudaStream_t st,
                                const float* lse_in, int cluster, int tpc);
+// The pruning layer's causal attention (O and the row lse) with the text rows'
+// score a and its Eq. 8 statistics as a by-product when a_out is given.
+cudaError_t launch_attention(const LayoutArgs& la, const void* q, int64_t q_stride, const void* k,
+                             int64_t k_stride, const void* v, int64_t v_stride, void* o_out,
+                             int64_t o_stride, float* lse_out, float* a_out, float4* stats,
+                             uint32_t* counters, uint32_t* status, cudaStream_t st);
 // Persistent single-CTA-per-unit score kernel and its applicability tests.
 bool score_unit_fits(const LayoutArgs& la, int mode);
 bool score_unit_single_group(const LayoutArgs& la, int mode);

@@ -182,6 +182,30 @@ class Decision:
                                 len(src), src, dst, row_bytes, pos_ids, self.ws, self.ws_bytes,
                                 stream), "e2s_prune")
 
+    def attention(self, q_all: torch.Tensor, k: torch.Tensor, v: torch.Tensor,
+                  o_out: torch.Tensor, lse_out: Optional[torch.Tensor] = None,
+                  with_score: bool = True, stream=None) -> None:
+        """e2s_attention: the layer's causal attention over q_all [L, sum_T, H, d]
+        (every row), into o_out (same shape) and lse_out [L, H, sum_T]; with
+        with_score, the decision's score into self.a as a by-product."""
+        b = self.batch
+        e2s.check(e2s.e2s_attention(b.layout, q_all, b.H * b.d, k, b.H_kv * b.d, v,
+                                    b.H_kv * b.d, o_out, b.H * b.d, lse_out,
+                                    self.a if with_score else None, self.ws, self.ws_bytes,
+                                    stream), "e2s_attention")
+
+    def decide_attn(self, q_all: torch.Tensor, k: torch.Tensor, v: torch.Tensor,
+                    o_out: torch.Tensor, lse_out: Optional[torch.Tensor] = None,
+                    prior: Optional[torch.Tensor] = None, cand: Optional[torch.Tensor] = None,
+                    stream=None) -> None:
+        """e2s_decide_attn: the layer's attention, then the decision from its score."""
+        b = self.batch
+        e2s.check(e2s.e2s_decide_attn(b.layout, self.params, q_all, b.H * b.d, k, b.H_kv * b.d,
+                                      v, b.H_kv * b.d, o_out, b.H * b.d, lse_out, cand, prior,
+                                      self.a, self.mass, self.fused, self.q, self.keep_count,
+                                      self.keep_off, self.sum_keep, self.keep_idx, self.q_tilde,
+                                      self.ws, self.ws_bytes, stream), "e2s_decide_attn")
+
     def run(self, q_text: torch.Tensor, k: torch.Tensor, stream=None) -> None:
         """The decision itself: score + fuse + select (e2s_decide)."""
         self.decide(q_text, k, stream=stream)

@@ -93,6 +93,11 @@ _SIGS = {
     "e2s_read_status": (ctypes.c_int, [_vp, _vp]),
     "e2s_clear_status": (ctypes.c_int, [_vp, _vp]),
     "e2s_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "e2s_attention": (ctypes.c_int, [_LP, _vp, _i64, _vp, _i64, _vp, _i64, _vp, _i64, _vp,
+                                      _vp, _vp, _sz, _vp]),
+    "e2s_decide_attn": (ctypes.c_int, [_LP, _PP, _vp, _i64, _vp, _i64, _vp, _i64, _vp, _i64,
+                                        _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _vp,
+                                        _vp, _vp, _sz, _vp]),
     "e2s_selftest_bounded_wait": (ctypes.c_int, [_i32, _i64, _vp, _vp]),
     "e2s_version": (ctypes.c_int32, []),
 }
@@ -213,6 +218,25 @@ def e2s_fuse(layout, params_, a, cand, prior, mass_out, fused_out, q_out, ws, ws
 def e2s_fuse_select(layout, params_, a, cand, prior, mass_out, fused_out, q_out, keep_count,
                     keep_off, sum_keep, keep_idx, q_tilde_out, ws, ws_bytes, stream=None) -> int:
     return lib.e2s_fuse_select(_ref(layout), _ref(params_), _ptr(a), _ptr(cand), _ptr(prior),
+                               _ptr(mass_out), _ptr(fused_out), _ptr(q_out), _ptr(keep_count),
+                               _ptr(keep_off), sum_keep, _ptr(keep_idx), _ptr(q_tilde_out),
+                               _ptr(ws), ws_bytes, _stream(stream))
+
+
+def e2s_attention(layout, q, q_row_stride, k, k_row_stride, v, v_row_stride, o_out,
+                  o_row_stride, lse_out, a_out, ws, ws_bytes, stream=None) -> int:
+    return lib.e2s_attention(_ref(layout), _ptr(q), q_row_stride, _ptr(k), k_row_stride, _ptr(v),
+                             v_row_stride, _ptr(o_out), o_row_stride, _ptr(lse_out), _ptr(a_out),
+                             _ptr(ws), ws_bytes, _stream(stream))
+
+
+def e2s_decide_attn(layout, params_, q, q_row_stride, k, k_row_stride, v, v_row_stride, o_out,
+                    o_row_stride, lse_out, cand, prior, a_out, mass_out, fused_out, q_out,
+                    keep_count, keep_off, sum_keep, keep_idx, q_tilde_out, ws, ws_bytes,
+                    stream=None) -> int:
+    return lib.e2s_decide_attn(_ref(layout), _ref(params_), _ptr(q), q_row_stride, _ptr(k),
+                               k_row_stride, _ptr(v), v_row_stride, _ptr(o_out), o_row_stride,
+                               _ptr(lse_out), _ptr(cand), _ptr(prior), _ptr(a_out),
                                _ptr(mass_out), _ptr(fused_out), _ptr(q_out), _ptr(keep_count),
                                _ptr(keep_off), sum_keep, _ptr(keep_idx), _ptr(q_tilde_out),
                                _ptr(ws), ws_bytes, _stream(stream))

@@ -272,6 +272,25 @@ def make_inputs(spec: Spec, *, with_payload: bool = True) -> Inputs:
                   keep, keep_off, q, k, v, hid, salient)
 
 
+def full_queries(inp: Inputs) -> np.ndarray:
+    """Queries of every row of every image, [L, sum T, H, d] bf16 bits, for the
+    layer's own attention pass: the text rows are inp.q_text (so the text
+    rows' scores are those of the decision), the system and visual rows are
+    i.i.d. normal with variance d**-0.5 from a stream of their own per image
+    (seed 1000 * config + image + 2**41)."""
+    s = inp.spec
+    q = np.empty((s.L, int(inp.tok_off[-1]), s.H, s.d), dtype=np.uint16)
+    for b in range(s.B):
+        rng = np.random.Generator(np.random.PCG64(1000 * s.cfg_id + b + (1 << 41)))
+        t0, S, NV, NT = int(inp.tok_off[b]), int(inp.n_sys[b]), int(inp.n_vis[b]), int(inp.n_text[b])
+        x0 = int(inp.text_off[b])
+        for l in range(s.L):
+            q[l, t0:t0 + S + NV] = bf16_bits(
+                rng.standard_normal((S + NV, s.H, s.d), dtype=np.float32) * np.float32(SIGMA))
+            q[l, t0 + S + NV:t0 + S + NV + NT] = inp.q_text[l, x0:x0 + NT]
+    return q
+
+
 def custom_spec(name: str, images: Sequence[ImageSpec], *, L: int = 2, H: int = 4, H_kv: int = 4,
                 hidden: int = 0, cfg_id: int = 9) -> Spec:
     """A free-form spec for edge-case tests (small heads, odd grids, K=0 ...)."""

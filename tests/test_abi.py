@@ -57,7 +57,7 @@ def test_workspace_size_and_versions():
     # status word, one float4 per (image, layer, head), 64 cell keys + a counter per image
     assert n == 256 + ((1 * 2 * 32 * 16 + 255) // 256) * 256 + ((1 * 129 * 4 + 255) // 256) * 256
     assert e2s.e2s_workspace_size(_layout(e2s, d=64), e2s.params()) == 0
-    assert e2s.e2s_version() == 102
+    assert e2s.e2s_version() == 103
     assert e2s.e2s_status_string(e2s.E2S_ERR_TIMEOUT) == "E2S_ERR_TIMEOUT"
     assert e2s.e2s_status_string(99) == "E2S_ERR_UNKNOWN"
 
@@ -228,3 +228,24 @@ def test_selftest_bounded_wait_host_validation():
     assert e2s.e2s_selftest_bounded_wait(0, 50_000_000, 0x1010) == e2s.E2S_ERR_WORKSPACE
     assert e2s.e2s_selftest_bounded_wait(0, 10, 0x1000) == e2s.E2S_ERR_INVALID_ARG
     assert e2s.e2s_selftest_bounded_wait(0, 3_000_000_000, 0x1000) == e2s.E2S_ERR_INVALID_ARG
+
+
+def test_attention_host_validation():
+    e2s = _lib()
+    lay = _layout(e2s)
+    ws = 0x100000
+    wsb = e2s.e2s_workspace_size(lay, e2s.params())
+    fake = 0x2000
+    # every call below fails host validation, so nothing is launched
+    assert e2s.e2s_attention(lay, None, 4096, fake, 4096, fake, 4096, fake, 4096, None, None,
+                             ws, wsb) == e2s.E2S_ERR_INVALID_ARG
+    assert e2s.e2s_attention(lay, fake, 4000, fake, 4096, fake, 4096, fake, 4096, None, None,
+                             ws, wsb) == e2s.E2S_ERR_SHAPE
+    assert e2s.e2s_attention(lay, fake + 8, 4096, fake, 4096, fake, 4096, fake, 4096, None, None,
+                             ws, wsb) == e2s.E2S_ERR_ALIGNMENT
+    assert e2s.e2s_attention(_layout(e2s, max_text=129, max_T=700, sum_T=700, sum_text=129),
+                             fake, 4096, fake, 4096, fake, 4096, fake, 4096, None, fake, ws,
+                             wsb * 2) == e2s.E2S_ERR_UNSUPPORTED
+    assert e2s.e2s_decide_attn(lay, e2s.params(score_mode=e2s.E2S_SCORE_EQ1), fake, 4096, fake,
+                               4096, fake, 4096, fake, 4096, None, None, None, fake, None, fake,
+                               fake, fake, fake, 0, None, None, ws, wsb) == e2s.E2S_ERR_UNSUPPORTED
