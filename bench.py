@@ -611,6 +611,54 @@ def measure_batched(name: str, dev, peaks: dict, steps: int) -> dict:
     return out
 
 
+def attention_pass_entry(T: Timing, w: Workload, n: int, decision_us: float, peaks) -> dict:
+    """The pruning layer's own attention (e2s_attention, every row's O and lse)
+    alone, with the decision's score as a by-product, and with the whole
+    decision after it (e2s_decide_attn); L2 flushed before every replay."""
+    import torch
+
+    from paper_2608_23253_gb300 import e2s, synth
+    from paper_2608_23253_gb300.decision import Decision, bf16_tensor
+    dev = w.q.device
+    s, b = w.s, w.batch
+    q_all = bf16_tensor(synth.full_queries(w.inp), dev)
+    o = torch.empty_like(q_all)
+    lse = torch.empty((s.L, s.H, b.sum_T), dtype=torch.float32, device=dev)
+    dx = Decision(b, w.inp.keep, e2s.params())
+    st = T.stream
+    calls = {"attention": lambda: dx.attention(q_all, w.k, w.v, o, lse, with_score=False,
+                                               stream=st),
+             "attention_with_score": lambda: dx.attention(q_all, w.k, w.v, o, lse, stream=st),
+             "attention_then_decision": lambda: dx.decide_attn(q_all, w.k, w.v, o, lse,
+                                                               stream=st)}
+    out = {}
+    with torch.cuda.stream(st):
+        for fn in calls.values():
+            fn()
+        st.synchronize()
+        e2s.check(dx.status(st), "device status (attention pass)")
+        for name, fn in calls.items():
+            gx = T.capture([fn])
+            for _ in range(3):
+                T.run(gx)
+            out[name] = statistics.mean(T.run(gx) for _ in range(n)) * 1e3
+    # causal pairs (row, visible key) of every image; QK^T and PV, 2 flops each
+    pairs = sum((t * (t + 1)) // 2 for t in (w.inp.n_sys + w.inp.n_vis + w.inp.n_text))
+    flops = 2.0 * 2.0 * s.H * s.d * s.L * pairs
+    tf = (peaks or {}).get("bf16_tflops") or 1900.0
+    return {"attention_us": out["attention"],
+            "attention_with_score_us": out["attention_with_score"],
+            "score_extra_us": out["attention_with_score"] - out["attention"],
+            "attention_then_decision_us": out["attention_then_decision"],
+            "separate_score_then_decision_us": decision_us,
+            "attention_TFLOP/s": flops / (out["attention"] * 1e-6) / 1e12,
+            "attention_frac_of_bf16_peak": flops / (out["attention"] * 1e-6) / 1e12 / tf,
+            "note": "e2s_attention over the pruning layer's 3 evidence layers (all 675 rows, "
+                    "causal, O and lse of every row); with_score adds the text rows' score a "
+                    "and its statistics in the same launch; attention_then_decision = "
+                    "e2s_decide_attn; separate = e2s_decide (its own score kernel)"}
+
+
 def run_ours(args, world, rank, local):
     import torch
 
@@ -832,6 +880,7 @@ def run_ours(args, world, rank, local):
                        "step_us": statistics.mean(step_ms) * 1e3,
                        "decision_us": decision_us, "decide_kernel_us": stage_ms["decide"] * 1e3}
         line["ablations"] = abl
+        line["attention_pass"] = attention_pass_entry(T, w, n_stage, decision_us, peaks)
     if extras and flags == 0:
         line["batched"] = {name: measure_batched(name, dev, peaks, max(args.steps // 10, 20))
                            for name in ("cfg2", "cfg3", "cfg4") if name != args.workload}
