@@ -10,10 +10,14 @@
 // way; query tile i attends to key tiles i .. n-1 (tile i is the diagonal).
 // Per key tile, in ascending key order:
 //   MMA   S = Q K^T (text rows on the TMEM lanes, M = N = 128), double-buffered;
-//   softmax warps (one thread per row): masked row maximum, rescale factor
-//         alpha = 2^(m_old - m_new), P = 2^(s - m_new) rounded to bf16 into
-//         shared memory (the K-major, 128-byte-swizzled A operand), running
-//         row sum; the O accumulator is rescaled in TMEM when some alpha != 1;
+//   softmax warps (two per lane quarter, 64 columns each; a row's two halves
+//         exchange their maxima and, at the end, their sums through shared
+//         memory): masked row maximum; the row's reference maximum m moves
+//         only when the tile exceeds it by more than kLazy (log2 units), so P =
+//         2^(s - m) <= 2^kLazy and O needs rescaling (by 2^(m_old - m_new), in
+//         TMEM, after the previous P V) only then; P in bf16 into one of two
+//         shared-memory buffers (the K-major, 128-byte-swizzled A operand), so
+//         the softmax of a tile overlaps the previous tile's P V;
 //   MMA   O += P V (V as the MN-major B operand straight from its TMA tile).
 // Then O / l goes out in bf16 and lse = (m + log2 l) ln 2 per row.  Tile 0's
 // CTA then has the final normaliser of every text row and, when the score is
@@ -22,8 +26,9 @@
 // lane-local, and the Eq. 8 statistics of the unit's visual scores follow
 // from the same lanes -- no other kernel reads K for the decision.
 //
-// Warp roles (192 threads): warp 0 TMA producer, warp 1 TMEM allocator and MMA
-// issuer, warps 2-5 softmax / epilogue (warp w reads TMEM lane quarter w % 4).
+// Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator and MMA
+// issuer, warps 2-9 softmax / epilogue (warp w reads TMEM lane quarter w % 4,
+// columns 64 * ((w - 2) / 4) .. of each tile).
 // Every mbarrier wait is bounded and reports E2S_ERR_TIMEOUT.
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -43,7 +48,8 @@ namespace {
 constexpr int kTile = 128;                    // query rows and keys per tile
 constexpr int kHalfBytes = kTile * 128;       // 128 rows x 64 bf16
 constexpr int kTileBytes = 2 * kHalfBytes;
-constexpr int kEpiWarps = 4;
+constexpr int kEpiWarps = 8;
+constexpr float kLazy = 8.f;                  // log2 headroom of the reference maximum
 constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr int kThreads = 64 + kEpiThreads;
 constexpr uint32_t kColsS = 128;              // TMEM columns per S buffer
@@ -68,7 +74,7 @@ struct AttnArgs {
 };
 
 struct APlan {
-  uint32_t q, k, v, p, bars, slot, nlse, red, total;
+  uint32_t q, k, v, p, bars, slot, nlse, xch, red, total;
 };
 
 __host__ __device__ inline APlan attn_plan() {
@@ -76,12 +82,13 @@ __host__ __device__ inline APlan attn_plan() {
   s.q = 0;
   s.k = kTileBytes;                 // 2 stages
   s.v = s.k + 2 * kTileBytes;       // 2 stages
-  s.p = s.v + 2 * kTileBytes;       // P: two 64-key halves of 128 rows
-  s.bars = s.p + kTileBytes;
-  s.slot = s.bars + 8u * 16u;
+  s.p = s.v + 2 * kTileBytes;       // 2 buffers of P, each two 64-key halves of 128 rows
+  s.bars = s.p + 2 * kTileBytes;
+  s.slot = s.bars + 8u * 20u;
   s.nlse = (s.slot + 16u + 15u) & ~15u;   // float [128]
-  s.red = s.nlse + kTile * 4u;            // float4 [kEpiWarps]
-  s.total = s.red + kEpiWarps * 16u;
+  s.xch = s.nlse + kTile * 4u;            // float [2][128]: the two column halves of a row
+  s.red = s.xch + 2 * kTile * 4u;         // float4 [4]
+  s.total = s.red + 4 * 16u;
   return s;
 }
 
@@ -152,10 +159,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* v_free = v_full + 2;     // [2]
   uint64_t* s_full = v_free + 2;     // [2]
   uint64_t* s_free = s_full + 2;     // [2]
-  uint64_t* p_ready = s_free + 2;    // P of the current tile written, O rescaled
-  uint64_t* pv_done = p_ready + 1;   // the last O += P V is complete
+  uint64_t* p_ready = s_free + 2;    // [2] P buffer b written (and O rescaled if needed)
+  uint64_t* pv_done = p_ready + 2;   // [2] the O += P V reading P buffer b is complete
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + plan.slot);
   float* nlse = reinterpret_cast<float*>(smem + plan.nlse);
+  float* xch = reinterpret_cast<float*>(smem + plan.xch);
   float4* red = reinterpret_cast<float4*>(smem + plan.red);
 
   const LayoutArgs& la = p.la;
@@ -181,9 +189,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::mbar_init(v_free + i, 1);
       ptx::mbar_init(s_full + i, 1);
       ptx::mbar_init(s_free + i, kEpiWarps);
+      ptx::mbar_init(p_ready + i, kEpiWarps);
+      ptx::mbar_init(pv_done + i, 1);
     }
-    ptx::mbar_init(p_ready, kEpiWarps);
-    ptx::mbar_init(pv_done, 1);
     ptx::fence_barrier_init();
     ptx::fence_proxy_async_smem();
   }
@@ -230,7 +238,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       if (!ptx::mbar_wait(q_full, 0, limit, p.status)) limit = kWaitNsAfterFault;
       const uint32_t q_base = ptx::smem_addr(q_sm);
-      const uint32_t p_base = ptx::smem_addr(p_sm);
       const uint32_t idesc_s = ptx::idesc_bf16_f32(kTile, kTile);
       const uint32_t idesc_pv = ptx::idesc_bf16_f32(kTile, 128) | (1u << 16);   // B MN-major
       int lk = 0, lv = 0;
@@ -255,10 +262,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++lk;
       };
       auto pv = [&](int x) {
-        if (!ptx::mbar_wait(p_ready, x & 1, limit, p.status)) limit = kWaitNsAfterFault;
+        const int pb = x & 1;
+        if (!ptx::mbar_wait(p_ready + pb, (x >> 1) & 1, limit, p.status)) limit = kWaitNsAfterFault;
         const int s = lv & 1;
         if (!ptx::mbar_wait(v_full + s, (lv >> 1) & 1, limit, p.status)) limit = kWaitNsAfterFault;
         ptx::tc_fence_after();
+        const uint32_t p_base = ptx::smem_addr(p_sm + pb * kTileBytes);
         const uint32_t v_base = ptx::smem_addr(v_sm + s * kTileBytes);
 #pragma unroll
         for (int ks = 0; ks < 8; ++ks) {
@@ -268,7 +277,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           ptx::mma_bf16(tmem + kColO, pd, vd, idesc_pv, (x > 0 || ks > 0) ? 1u : 0u);
         }
         ptx::mma_commit(v_free + s);
-        ptx::mma_commit(pv_done);
+        ptx::mma_commit(pv_done + pb);
         ++lv;
       };
       for (int jj = 0; jj < nk; ++jj) {
@@ -283,94 +292,114 @@ __global__ void __launch_bounds__(kThreads, 1)
         qk(nk + vt, q_base + (uint32_t)(kTile - ntp2) * 128u, idesc_a, true);
     }
   } else {
-    // ================= softmax / epilogue: one thread per TMEM lane (query row)
+    // ================= softmax / epilogue: lane quarter q4, columns of half ch
+    const int ew = warp - 2;
     const int q4 = warp & 3;
-    const int r = q4 * 32 + lane;
+    const int ch = ew >> 2;                        // 0 or 1: tile columns 64 ch .. 64 ch + 63
+    const int r = q4 * 32 + lane;                  // TMEM lane (query row of the tile)
     const uint32_t lane_base = (uint32_t)(q4 * 32) << 16;
-    const int qp = g.row0 + r;            // image position of this row
+    const uint32_t pair_bar = 2u + (uint32_t)q4;   // the two warps of this lane quarter
+    const int qp = g.row0 + r;                     // image position of this row
     const bool rvalid = qp >= 0;
-    float m = kNegBig, lsum = 0.f;
+    float m = kNegBig, lsum = 0.f;                 // reference maximum and this half's sum
     for (int jj = 0; jj < nk; ++jj) {
-      const int sb = jj & 1;
+      const int sb = jj & 1, pb = jj & 1;
       const int kbase = g.T - kTile * (g.nq - jj);   // image position of the tile's key 0
       const int c_lo = max(0, -kbase), c_hi = min(kTile - 1, qp - kbase);
-      const bool full = c_lo == 0 && c_hi == kTile - 1;
+      const int c0 = 64 * ch;
+      const bool full = c_lo <= c0 && c_hi >= c0 + 63;
       if (!ptx::mbar_wait(s_full + sb, (jj >> 1) & 1, limit, p.status)) limit = kWaitNsAfterFault;
       ptx::tc_fence_after();
-      const uint32_t sa = tmem + lane_base + (uint32_t)sb * kColsS;
-      // pass 1: masked row maximum of the tile
-      float cmax = kNegBig;
-      for (int c16 = 0; c16 < kTile; c16 += 16) {
+      const uint32_t sa = tmem + lane_base + (uint32_t)sb * kColsS + (uint32_t)c0;
+      // pass 1: masked maximum of this half, then of the row (the other half's
+      // through shared memory)
+      float hmax = kNegBig;
+      for (int c16 = 0; c16 < 64; c16 += 16) {
         float x[16];
         ptx::tmem_ld16(sa + c16, x);
         if (full) {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) cmax = fmaxf(cmax, x[i]);
+          for (int i = 0; i < 16; ++i) hmax = fmaxf(hmax, x[i]);
         } else {
 #pragma unroll
           for (int i = 0; i < 16; ++i)
-            if (c16 + i >= c_lo && c16 + i <= c_hi) cmax = fmaxf(cmax, x[i]);
+            if (c0 + c16 + i >= c_lo && c0 + c16 + i <= c_hi) hmax = fmaxf(hmax, x[i]);
         }
       }
-      const float mnew = fmaxf(m, cmax > 0.5f * kNegBig ? cmax * p.scale_log2 : kNegBig);
-      const float alpha = fast_ex2(m - mnew);
-      // the previous O += P V must be complete before P is overwritten and O rescaled
-      if (jj >= 1 && !ptx::mbar_wait(pv_done, (jj - 1) & 1, limit, p.status))
+      xch[ch * kTile + r] = hmax;
+      ptx::named_bar(pair_bar, 64);
+      const float tmax = fmaxf(xch[r], xch[kTile + r]);
+      ptx::named_bar(pair_bar, 64);   // xch is rewritten only after both halves read it
+      const float tm = tmax > 0.5f * kNegBig ? tmax * p.scale_log2 : kNegBig;
+      // the reference maximum moves only by more than kLazy (or from empty)
+      const bool move = tm > m + kLazy || (m <= 0.5f * kNegBig && tm > 0.5f * kNegBig);
+      const float mnew = move ? tm : m;
+      const float alpha = move ? fast_ex2(m - mnew) : 1.f;
+      if (jj >= 1 && __any_sync(0xffffffffu, move)) {
+        // O of these rows is rescaled once the previous P V is complete
+        const int pp = (jj - 1) & 1;
+        if (!ptx::mbar_wait(pv_done + pp, ((jj - 1) >> 1) & 1, limit, p.status))
+          limit = kWaitNsAfterFault;
+        ptx::tc_fence_after();
+        for (int c16 = 0; c16 < 64; c16 += 16) {
+          float x[16];
+          ptx::tmem_ld16(tmem + lane_base + kColO + (uint32_t)(c0 + c16), x);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) x[i] *= alpha;
+          ptx::tmem_st16(tmem + lane_base + kColO + (uint32_t)(c0 + c16), x);
+        }
+        ptx::tmem_wait_st();
+      }
+      // P buffer pb is free once the P V two tiles back is complete
+      if (jj >= 2 && !ptx::mbar_wait(pv_done + pb, ((jj >> 1) - 1) & 1, limit, p.status))
         limit = kWaitNsAfterFault;
-      ptx::tc_fence_after();
-      // pass 2: P = 2^(s - m) in bf16, K-major 128-byte-swizzled rows of the A operand
+      // pass 2: P = 2^(s - m) in bf16 into this half's 64-key half of the A operand
+      uint8_t* prow = p_sm + pb * kTileBytes + ch * kHalfBytes + r * 128;
       float acc = 0.f;
-      for (int c16 = 0; c16 < kTile; c16 += 16) {
+      for (int c16 = 0; c16 < 64; c16 += 16) {
         float x[16];
         ptx::tmem_ld16(sa + c16, x);
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const bool vis = full || (c16 + i >= c_lo && c16 + i <= c_hi);
+          const bool vis = full || (c0 + c16 + i >= c_lo && c0 + c16 + i <= c_hi);
           x[i] = vis ? fast_ex2(fmaf(x[i], p.scale_log2, -mnew)) : 0.f;
           acc += x[i];
         }
-        const int half = c16 >> 6;
 #pragma unroll
-        for (int ch = 0; ch < 2; ++ch) {
-          const int chunk = ((c16 & 63) >> 3) + ch;
+        for (int h8 = 0; h8 < 2; ++h8) {
+          const int chunk = (c16 >> 3) + h8;
           uint4 w;
-          w.x = pack_bf16(x[8 * ch + 0], x[8 * ch + 1]);
-          w.y = pack_bf16(x[8 * ch + 2], x[8 * ch + 3]);
-          w.z = pack_bf16(x[8 * ch + 4], x[8 * ch + 5]);
-          w.w = pack_bf16(x[8 * ch + 6], x[8 * ch + 7]);
-          *reinterpret_cast<uint4*>(p_sm + half * kHalfBytes + r * 128 +
-                                    ((chunk ^ (r & 7)) << 4)) = w;
+          w.x = pack_bf16(x[8 * h8 + 0], x[8 * h8 + 1]);
+          w.y = pack_bf16(x[8 * h8 + 2], x[8 * h8 + 3]);
+          w.z = pack_bf16(x[8 * h8 + 4], x[8 * h8 + 5]);
+          w.w = pack_bf16(x[8 * h8 + 6], x[8 * h8 + 7]);
+          *reinterpret_cast<uint4*>(prow + ((chunk ^ (r & 7)) << 4)) = w;
         }
       }
       lsum = lsum * alpha + acc;
       m = mnew;
-      ptx::tc_fence_before();
-      __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(s_free + sb);
-      // rescale the O accumulator of this row (the first tile overwrites it)
-      if (jj >= 1 && !__all_sync(0xffffffffu, alpha == 1.f)) {
-        for (int c16 = 0; c16 < 128; c16 += 16) {
-          float x[16];
-          ptx::tmem_ld16(tmem + lane_base + kColO + c16, x);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) x[i] *= alpha;
-          ptx::tmem_st16(tmem + lane_base + kColO + c16, x);
-        }
-        ptx::tmem_wait_st();
-      }
       ptx::fence_proxy_async_smem();   // P's generic-proxy stores -> the tensor core
       ptx::tc_fence_before();
       __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(p_ready);
+      if (lane == 0) {
+        ptx::mbar_arrive(s_free + sb);
+        ptx::mbar_arrive(p_ready + pb);
+      }
     }
-    // ---- O / l and the row normaliser
-    if (!ptx::mbar_wait(pv_done, (nk - 1) & 1, limit, p.status)) limit = kWaitNsAfterFault;
+    // ---- O / l and the row normaliser (the two halves' sums meet in xch)
+    xch[ch * kTile + r] = lsum;
+    ptx::named_bar(pair_bar, 64);
+    const float ltot = xch[r] + xch[kTile + r];
+    const int pl = (nk - 1) & 1;
+    if (!ptx::mbar_wait(pv_done + pl, ((nk - 1) >> 1) & 1, limit, p.status))
+      limit = kWaitNsAfterFault;
     ptx::tc_fence_after();
-    const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
-    uint16_t* orow = p.o_out + (int64_t)(base_row + qp) * p.o_stride + (int64_t)g.h * 128;
-    for (int c16 = 0; c16 < 128; c16 += 16) {
+    const float inv = ltot > 0.f ? 1.f / ltot : 0.f;
+    uint16_t* orow =
+        p.o_out + (int64_t)(base_row + qp) * p.o_stride + (int64_t)g.h * 128 + 64 * ch;
+    for (int c16 = 0; c16 < 64; c16 += 16) {
       float x[16];
-      ptx::tmem_ld16(tmem + lane_base + kColO + c16, x);
+      ptx::tmem_ld16(tmem + lane_base + kColO + (uint32_t)(64 * ch + c16), x);
       if (rvalid) {
         uint4 w0, w1;
         w0.x = pack_bf16(x[0] * inv, x[1] * inv);
@@ -385,14 +414,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         *reinterpret_cast<uint4*>(orow + c16 + 8) = w1;
       }
     }
-    const float lse2 = lsum > 0.f ? m + __log2f(lsum) : -kNegBig;
-    if (rvalid && p.lse_out != nullptr)
-      p.lse_out[((int64_t)g.l * la.H + g.h) * la.sum_T + g.t0 + qp] = lse2 * kLn2;
-    nlse[r] = -lse2;
+    const float lse2 = ltot > 0.f ? m + __log2f(ltot) : -kNegBig;
+    if (ch == 0) {
+      if (rvalid && p.lse_out != nullptr)
+        p.lse_out[((int64_t)g.l * la.H + g.h) * la.sum_T + g.t0 + qp] = lse2 * kLn2;
+      nlse[r] = -lse2;
+    }
     if (sweep) {
       // ---- the score from the final row normalisers: keys on the lanes,
-      // column c <-> tile row kTile - ntp2 + c <-> text row c - (ntp2 - NT)
-      ptx::named_bar(1, kEpiThreads);
+      // column c <-> tile row kTile - ntp2 + c <-> text row c - (ntp2 - NT);
+      // the two warps of a lane quarter take alternate 16-column chunks
+      ptx::named_bar(1, kEpiThreads);   // nlse complete, xch free
       const int c_text = ntp2 - g.NT;
       const float inv_nt = 1.f / (float)g.NT;
       float st_s = 0.f, st_m = kNegBig, st_e = 0.f;
@@ -401,9 +433,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!ptx::mbar_wait(s_full + sb, (jj >> 1) & 1, limit, p.status))
           limit = kWaitNsAfterFault;
         ptx::tc_fence_after();
-        const int key = kTile * vt + r;   // visual index of this lane's key
         float acc = 0.f;
-        for (int c16 = 0; c16 < ntp2; c16 += 16) {
+        for (int c16 = 16 * ch; c16 < ntp2; c16 += 32) {
           float x[16];
           ptx::tmem_ld16(tmem + lane_base + (uint32_t)sb * kColsS + c16, x);
 #pragma unroll
@@ -414,28 +445,34 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tc_fence_before();
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(s_free + sb);
-        if (key < g.NV) {
-          const float a = acc * inv_nt;
+        xch[ch * kTile + r] = acc;
+        ptx::named_bar(pair_bar, 64);
+        const int key = kTile * vt + r;   // visual index of this lane's key
+        if (ch == 0 && key < g.NV) {
+          const float a = (xch[r] + xch[kTile + r]) * inv_nt;
           p.a_out[((size_t)g.l * la.H + g.h) * (size_t)la.sum_vis + g.v0 + key] = a;
           const float al = a * kLog2e, mn = fmaxf(st_m, al);
           st_e = st_e * fast_ex2(st_m - mn) + fast_ex2(al - mn);
           st_m = mn;
           st_s += a;
         }
+        ptx::named_bar(pair_bar, 64);   // xch is rewritten by the next tile
       }
+      if (ch == 0) {
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const float s2 = __shfl_xor_sync(0xffffffffu, st_s, o);
-        const float m2 = __shfl_xor_sync(0xffffffffu, st_m, o);
-        const float e2 = __shfl_xor_sync(0xffffffffu, st_e, o);
-        st_s += s2;
-        lse_merge(st_m, st_e, m2, e2);
+        for (int o = 16; o > 0; o >>= 1) {
+          const float s2 = __shfl_xor_sync(0xffffffffu, st_s, o);
+          const float m2 = __shfl_xor_sync(0xffffffffu, st_m, o);
+          const float e2 = __shfl_xor_sync(0xffffffffu, st_e, o);
+          st_s += s2;
+          lse_merge(st_m, st_e, m2, e2);
+        }
+        if (lane == 0) red[q4] = make_float4(st_s, st_m, st_e, 0.f);
       }
-      if (lane == 0) red[q4] = make_float4(st_s, st_m, st_e, 0.f);
       ptx::named_bar(1, kEpiThreads);
-      if (r == 0) {   // the four lane quarters in order
+      if (r == 0 && ch == 0) {   // the four lane quarters in order
         float S = 0.f, M = kNegBig, E = 0.f;
-        for (int w = 0; w < kEpiWarps; ++w) {
+        for (int w = 0; w < 4; ++w) {
           S += red[w].x;
           lse_merge(M, E, red[w].y, red[w].z);
         }
@@ -477,7 +514,13 @@ cudaError_t launch_attention(const LayoutArgs& la, const void* q, int64_t q_stri
       !make_score_map(&tmK, k, la.H_kv, (int64_t)la.L * la.sum_T, k_stride, kTile) ||
       !make_score_map(&tmV, v, la.H_kv, (int64_t)la.L * la.sum_T, v_stride, kTile))
     return cudaErrorInvalidValue;
-  const size_t smem = attn_plan().total + 1024;
+  const size_t smem = attn_plan().total + 1024;   // + alignment slack
+  int dev = 0, optin = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (e != cudaSuccess) return e;
+  if ((size_t)optin < smem) return cudaErrorInvalidConfiguration;
   return launch_kernel(attn_kernel, dim3((unsigned)(p.units * n_qt)), dim3(kThreads), smem, st,
                        0, false, tmQ, tmK, tmV, p);
 }
