@@ -675,6 +675,12 @@ def run_ours(args, world, rank, local):
     w = Workload(args.workload, dev, flags)
     inp, s, batch, dec = w.inp, w.s, w.batch, w.dec
     stream = T.stream
+    if args.attention_only:
+        # the pruning layer's attention pass alone (e2s_attention and
+        # e2s_decide_attn), for profiling: one JSON object, no headline line
+        print(json.dumps({"workload": args.workload, "attention_pass": attention_pass_entry(
+            T, w, max(args.steps, 3), None, measured_peaks())}), flush=True)
+        return
     step_call = lambda: w.prune(stream)   # noqa: E731
 
     with torch.cuda.stream(stream):
@@ -904,6 +910,8 @@ def main():
                          "or the flag word")
     ap.add_argument("--no-extras", action="store_true",
                     help="skip the batched, ablation and layer-comparator context keys")
+    ap.add_argument("--attention-only", action="store_true",
+                    help="time only the pruning layer's attention pass (for profiling)")
     args = ap.parse_args()
     if args.warmup < 3:
         raise SystemExit("--warmup must be >= 3")

@@ -105,8 +105,9 @@ typedef struct {
 /* Bytes of workspace every call below needs: the status word, one float4 of
  * normalisation statistics per (image, layer, head) written by e2s_score and
  * e2s_decide, and one arrival counter per image (e2s_decide).  The workspace
- * must be 256-byte aligned and its first 4 bytes zero before the first call
- * (see e2s_clear_status); the rest needs no initialisation. */
+ * must be 256-byte aligned and its first 16 bytes zero before the first call
+ * (e2s_clear_status zeroes them; bytes 4..15 hold the attention kernel's item
+ * counter, which every call leaves zero); the rest needs no initialisation. */
 size_t e2s_workspace_size(const e2s_layout* layout, const e2s_params* params);
 
 /* Text-to-visual score (Sec. 3.1, Eq. 1; Algorithm 1 "Compute a_{l,h,n}").
@@ -169,7 +170,9 @@ e2s_status e2s_score_lse(const e2s_layout* layout, const e2s_params* params,
  * Pointers 16-byte aligned (lse_out, a_out 4), strides multiples of 8 and at
  * least H*d (q, o) or H_kv*d (k, v).  P is rounded to bf16 before P V, as in
  * flash-attention forwards, so O carries bf16 rounding of the weights; lse
- * and a are computed from the fp32 logits. */
+ * and a are computed from the fp32 logits.  The CTAs share an item counter in
+ * the workspace (bytes 4..15, zero before and after the call), so calls that
+ * may run concurrently need separate workspaces. */
 e2s_status e2s_attention(const e2s_layout* layout, const void* q, int64_t q_row_stride,
                          const void* k, int64_t k_row_stride, const void* v, int64_t v_row_stride,
                          void* o_out, int64_t o_row_stride, float* lse_out, float* a_out,
@@ -357,7 +360,8 @@ e2s_status e2s_compact(const e2s_layout* layout, const int32_t* keep_idx,
  * error).  Does not clear it. */
 e2s_status e2s_read_status(const void* ws, void* stream);
 
-/* Zeroes the device status word (stream-ordered, asynchronous). */
+/* Zeroes the first 16 bytes of the workspace: the device status word and the
+ * attention kernel's item counter (stream-ordered, asynchronous). */
 e2s_status e2s_clear_status(void* ws, void* stream);
 
 /* Human-readable name of a status value (static string). */

@@ -8,10 +8,11 @@
 // aligned to the END of each image's sequence, so tile 0 holds the last 128
 // rows: every text row when N_T <= 128.  Key tiles are aligned the same way;
 // query tile i attends to key tiles i .. n-1 (tile i is the diagonal).  The
-// kernel is persistent: one CTA per SM walks the item list in passes of
-// alternating direction (tile 0 of every unit first: the heaviest items), so
-// TMEM and the barriers are set up once and the loads of the next item
-// overlap the end of the current one (two Q buffers).
+// kernel is persistent: one CTA per SM takes items in order (tile 0 of every
+// unit first: the heaviest items) from a counter shared by all CTAs, so TMEM
+// and the barriers are set up once, the CTAs stay balanced, and the loads of
+// the next item overlap the end of the current one.  K and V tiles have three
+// buffers each.
 // Per key tile, in ascending key order:
 //   MMA   S = Q K^T (query rows on the TMEM lanes, M = N = 128), two S buffers;
 //   softmax warps (two per lane quarter, 64 columns each): the 64 values come
@@ -31,9 +32,12 @@
 // lane-local, and the Eq. 8 statistics of the unit's visual scores follow
 // from the same lanes -- no other kernel reads K for the decision.
 //
-// Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator and MMA
-// issuer, warps 2-9 softmax / epilogue (warp w reads TMEM lane quarter w % 4,
-// columns 64 * ((w - 2) / 4) .. of each tile).  TMEM (512 columns): S buffers
+// Warp roles (384 threads): warp 0 issues O += P V, warp 1 allocates TMEM and
+// issues S = Q K^T, warps 2-9 softmax / epilogue (warp w reads TMEM lane
+// quarter w % 4, columns 64 * ((w - 2) / 4) .. of each tile), warp 10 loads K
+// and Q, warp 11 loads V.  A thread that issues MMAs shares its SM
+// sub-partition with two softmax warps; splitting the two MMA streams over two
+// sub-partitions keeps their issue from falling behind the tensor pipe.  TMEM (512 columns): S buffers
 // at 0 and 128, O at 256, the two P buffers (64 columns each) at 384 and 448.
 // Every mbarrier wait is bounded and reports E2S_ERR_TIMEOUT.
 #include <cuda.h>
@@ -57,7 +61,10 @@ constexpr int kTileBytes = 2 * kHalfBytes;
 constexpr int kEpiWarps = 8;
 constexpr float kLazy = 8.f;                  // log2 headroom of the reference maximum
 constexpr int kEpiThreads = 32 * kEpiWarps;
-constexpr int kThreads = 64 + kEpiThreads;
+// warp roles: the two MMA issuers sit on different SM sub-partitions (warp % 4)
+// so neither shares its issue slots with more than two softmax warps
+constexpr int kWarpPV = 0, kWarpQK = 1, kWarpLoadK = 10, kWarpLoadV = 11;
+constexpr int kThreads = 32 * 12;
 constexpr uint32_t kColsS = 128;              // TMEM columns per S buffer
 constexpr uint32_t kColO = 256;               // first TMEM column of the O accumulator
 constexpr uint32_t kColP = 384;               // two P buffers of 64 columns (bf16 pairs)
@@ -74,30 +81,34 @@ struct AttnArgs {
   float scale_log2;     // log2(e) / sqrt(d)
   uint16_t* o_out;      // [L][sum_T] rows of (H x d) bf16
   int64_t o_stride;     // elements between consecutive rows
+  int o_v8;             // o_out and its rows are 32-byte aligned: 32-byte stores
   float* lse_out;       // nullable [L][H][sum_T]
   float* a_out;         // nullable [L][H][sum_vis]
   float4* stats;        // per (image, layer, head), written with a_out
   uint32_t* counters;   // nullable: decision scratch to zero
+  uint32_t* sched;      // [0] items handed out after the first, [1] CTAs done (zero on entry)
   uint32_t* status;
 };
 
+constexpr int kStages = 3;           // K and V tile buffers each
+
 struct APlan {
-  uint32_t q, k, v, bars, slot, nlse, xch, xsum, red, total;
+  uint32_t q, k, v, bars, slot, nlse, xch, red, total;
 };
 
-constexpr int kBars = 22;
+constexpr int kRing = 4;             // item slots shared by the roles
+constexpr int kBars = 4 * kStages + 13 + 2 * kRing;
 
 __host__ __device__ inline APlan attn_plan() {
   APlan s;
-  s.q = 0;                          // 2 buffers
-  s.k = 2 * kTileBytes;             // 2 stages
-  s.v = s.k + 2 * kTileBytes;       // 2 stages
-  s.bars = s.v + 2 * kTileBytes;
-  s.slot = s.bars + 8u * kBars;
-  s.nlse = (s.slot + 16u + 15u) & ~15u;   // float [128]
-  s.xch = s.nlse + kTile * 4u;            // float [2][2][128]: row maxima by tile parity
-  s.xsum = s.xch + 4 * kTile * 4u;        // float [2][128]: row sums, score partials
-  s.red = s.xsum + 2 * kTile * 4u;        // float4 [4]
+  s.q = 0;
+  s.k = kTileBytes;
+  s.v = s.k + kStages * kTileBytes;
+  s.bars = s.v + kStages * kTileBytes;
+  s.slot = s.bars + 8u * kBars;           // TMEM address, softmax item [2], item ring [kRing]
+  s.nlse = (s.slot + 32u + 15u) & ~15u;   // float [128]
+  s.xch = s.nlse + kTile * 4u;            // float [2][128]: the two column halves of a row
+  s.red = s.xch + 2 * kTile * 4u;         // float4 [4]
   s.total = s.red + 4 * 16u;
   return s;
 }
@@ -120,6 +131,15 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 }
 
 __device__ __forceinline__ float neg_inf() { return __int_as_float(0xff800000); }
+
+// 32-byte global store (8 packed words).
+__device__ __forceinline__ void st_global_v8(void* p, uint32_t a0, uint32_t a1, uint32_t a2,
+                                             uint32_t a3, uint32_t a4, uint32_t a5, uint32_t a6,
+                                             uint32_t a7) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(a0),
+               "r"(a1), "r"(a2), "r"(a3), "r"(a4), "r"(a5), "r"(a6), "r"(a7)
+               : "memory");
+}
 
 // D (TMEM) (+)= A B with A read from TMEM (row i of A on lane i; for 16-bit
 // types two consecutive K elements per 32-bit column, the lower index in the
@@ -232,11 +252,26 @@ __device__ __forceinline__ AGeo attn_geo(const AttnArgs& p, int w) {
   return g;
 }
 
-// The k-th item of this CTA: passes over the item list in alternating
-// direction (increasing in k, so the walk ends at the first item >= items).
-__device__ __forceinline__ int attn_item(int k) {
-  const int G = (int)gridDim.x, c = (int)blockIdx.x;
-  return k * G + ((k & 1) ? G - 1 - c : c);
+// Item k of this CTA's walk, as the K-load warp published it in the ring
+// (-1: no more items, or the wait ran out).
+__device__ __forceinline__ int ring_item(int k, uint64_t* item_full, const volatile int* ring,
+                                         uint64_t& limit, uint32_t* status) {
+  const int slot = k % kRing;
+  if (!ptx::mbar_wait(item_full + slot, (k / kRing) & 1, limit, status)) {
+    limit = kWaitNsAfterFault;
+    return -1;
+  }
+  return ring[slot];
+}
+
+// Per item: nk + nv key tiles and S tiles (nv visual key tiles of the score
+// sweep), nk value tiles and P V accumulations.
+enum { kOpsQK = 0, kOpsPV = 1 };
+
+__device__ __forceinline__ int stream_ops(const AGeo& g, const AttnArgs& p, int kind) {
+  const int nk = g.nq - g.qt;
+  const int nv = p.a_out != nullptr && g.qt == 0 ? (g.NV + kTile - 1) / kTile : 0;
+  return kind == kOpsQK ? nk + nv : nk;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -249,22 +284,26 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* q_sm = smem + plan.q;
   uint8_t* k_sm = smem + plan.k;
   uint8_t* v_sm = smem + plan.v;
-  uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + plan.bars);   // [2]
-  uint64_t* q_free = q_full + 2;     // [2] every MMA reading Q buffer b is complete
-  uint64_t* k_full = q_free + 2;     // [2]
-  uint64_t* k_free = k_full + 2;     // [2]
-  uint64_t* v_full = k_free + 2;     // [2]
-  uint64_t* v_free = v_full + 2;     // [2]
-  uint64_t* s_full = v_free + 2;     // [2]
+  uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + plan.bars);
+  uint64_t* q_free = q_full + 1;             // every MMA reading Q is complete
+  uint64_t* k_full = q_free + 1;             // [kStages]
+  uint64_t* k_free = k_full + kStages;       // [kStages]
+  uint64_t* v_full = k_free + kStages;       // [kStages]
+  uint64_t* v_free = v_full + kStages;       // [kStages]
+  uint64_t* s_full = v_free + kStages;       // [2]
   uint64_t* s_free = s_full + 2;     // [2]
   uint64_t* p_ready = s_free + 2;    // [2] P buffer b written (and O rescaled if needed)
   uint64_t* pv_done = p_ready + 2;   // [2] the O += P V reading P buffer b is complete
   uint64_t* o_free = pv_done + 2;    // the item's O has been read out of TMEM
-  uint64_t* fin = o_free + 1;        // every MMA of the CTA is complete
+  uint64_t* fin = o_free + 1;        // every MMA of both issuers is complete
+  uint64_t* kick = fin + 1;          // the first item's Q and first key tile have landed
+  uint64_t* item_full = kick + 1;    // [kRing] ring slot written
+  uint64_t* item_free = item_full + kRing;   // [kRing] ring slot read by every role
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + plan.slot);
+  volatile int* sm_item = reinterpret_cast<volatile int*>(smem + plan.slot + 4);    // [2]
+  volatile int* ring = reinterpret_cast<volatile int*>(smem + plan.slot + 16);      // [kRing]
   float* nlse = reinterpret_cast<float*>(smem + plan.nlse);
   float* xch = reinterpret_cast<float*>(smem + plan.xch);
-  float* xsum = reinterpret_cast<float*>(smem + plan.xsum);
   float4* red = reinterpret_cast<float4*>(smem + plan.red);
 
   const LayoutArgs& la = p.la;
@@ -275,146 +314,203 @@ __global__ void __launch_bounds__(kThreads, 1)
       p.counters[i] = 0u;
 
   if (warp == 0 && lane == 0) {
-    for (int i = 0; i < 2; ++i) {
-      ptx::mbar_init(q_full + i, 1);
-      ptx::mbar_init(q_free + i, 1);
+    ptx::mbar_init(q_full, 1);
+    ptx::mbar_init(q_free, 1);
+    for (int i = 0; i < kStages; ++i) {
       ptx::mbar_init(k_full + i, 1);
       ptx::mbar_init(k_free + i, 1);
       ptx::mbar_init(v_full + i, 1);
       ptx::mbar_init(v_free + i, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
       ptx::mbar_init(s_full + i, 1);
       ptx::mbar_init(s_free + i, kEpiWarps);
       ptx::mbar_init(p_ready + i, kEpiWarps);
       ptx::mbar_init(pv_done + i, 1);
     }
     ptx::mbar_init(o_free, kEpiWarps);
-    ptx::mbar_init(fin, 1);
+    ptx::mbar_init(fin, 2);
+    ptx::mbar_init(kick, 1);
+    for (int i = 0; i < kRing; ++i) {
+      ptx::mbar_init(item_full + i, 1);
+      ptx::mbar_init(item_free + i, 4);   // V loads, both MMA issuers, the softmax group
+    }
     ptx::fence_barrier_init();
     ptx::fence_proxy_async_smem();
   }
-  if (warp == 1) ptx::tmem_alloc(tmem_slot, 512);
+  if (warp == kWarpQK) ptx::tmem_alloc(tmem_slot, 512);
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   uint64_t limit = kWaitNs;
 
-  if (warp == 0) {
-    // ================= TMA producer
+  if (warp == kWarpLoadK) {
+    // ================= the item walk and TMA of each item's key tiles (then
+    // the score sweep's visual key tiles) and its Q, which goes in once the
+    // previous item's last S = Q K^T is complete (after the item's first two
+    // key tiles).  A CTA's first item is its block index; the next ones come
+    // from one counter shared by all CTAs, in item order (the heaviest query
+    // tiles first), one item ahead, through the ring.  The first item's Q and
+    // first key tile go out alone, so that the first S is not queued behind
+    // every other load of the start.
     if (lane == 0) {
-      int it = 0, lk = 0, lv = 0;
-      auto load_k = [&](int krow, int kvh) {
-        const int s = lk & 1;
-        if (lk >= 2 && !ptx::mbar_wait(k_free + s, ((lk >> 1) - 1) & 1, limit, p.status))
+      int it = 0, lk = 0;
+      bool kicked = false;
+      auto publish = [&](int k, int w) {
+        const int slot = k % kRing;
+        if (k >= kRing && !ptx::mbar_wait(item_free + slot, (k / kRing - 1) & 1, limit, p.status))
           limit = kWaitNsAfterFault;
-        ptx::mbar_arrive_expect_tx(k_full + s, kTileBytes);
-        ptx::tma_load_3d(k_sm + s * kTileBytes, &tmK, k_full + s, 0, kvh, krow);
-        ptx::tma_load_3d(k_sm + s * kTileBytes + kHalfBytes, &tmK, k_full + s, 64, kvh, krow);
-        ++lk;
+        ring[slot] = w < p.items ? w : -1;
+        ptx::mbar_arrive(item_full + slot);
       };
-      for (int kk = 0;; ++kk) {
-        const int w = attn_item(kk);
-        if (w >= p.items) break;
+      publish(0, (int)blockIdx.x);
+      for (int k = 0;; ++k) {
+        const int w = ring[k % kRing];
+        if (w < 0) break;
+        const uint32_t nxt = atomicAdd(p.sched, 1u);   // published after this item's loads
+        const AGeo g = attn_geo(p, w);
+        if (g.work) {
+        const int nk = g.nq - g.qt;
+        const int n = stream_ops(g, p, kOpsQK);
+        const int base_row = g.l * la.sum_T + g.t0;   // row of image position 0 in the maps
+        for (int j = 0; j < n; ++j) {
+          if (it == 0 ? j == 0 : j == min(2, n - 1)) {
+            if (it >= 1 && !ptx::mbar_wait(q_free, (it - 1) & 1, limit, p.status))
+              limit = kWaitNsAfterFault;
+            ptx::mbar_arrive_expect_tx(q_full, kTileBytes);
+            ptx::tma_load_3d(q_sm, &tmQ, q_full, 0, g.h, base_row + g.row0);
+            ptx::tma_load_3d(q_sm + kHalfBytes, &tmQ, q_full, 64, g.h, base_row + g.row0);
+          }
+          const int s = lk % kStages;
+          if (lk >= kStages && !ptx::mbar_wait(k_free + s, (lk / kStages - 1) & 1, limit, p.status))
+            limit = kWaitNsAfterFault;
+          const int krow = j < nk ? base_row + g.T - kTile * (g.nq - j)
+                                  : base_row + g.S + kTile * (j - nk);
+          ptx::mbar_arrive_expect_tx(k_full + s, kTileBytes);
+          ptx::tma_load_3d(k_sm + s * kTileBytes, &tmK, k_full + s, 0, g.kvh, krow);
+          ptx::tma_load_3d(k_sm + s * kTileBytes + kHalfBytes, &tmK, k_full + s, 64, g.kvh, krow);
+          ++lk;
+          if (!kicked) {
+            // only this thread completes these phases, so the waits cannot alias
+            if (!ptx::mbar_wait(q_full, 0, limit, p.status)) limit = kWaitNsAfterFault;
+            if (!ptx::mbar_wait(k_full, 0, limit, p.status)) limit = kWaitNsAfterFault;
+            ptx::mbar_arrive(kick);
+            kicked = true;
+          }
+        }
+        ++it;
+        }
+        publish(k + 1, (int)(gridDim.x + nxt));
+      }
+      if (!kicked) ptx::mbar_arrive(kick);
+    }
+  } else if (warp == kWarpLoadV) {
+    // ================= TMA: each item's value tiles
+    if (lane == 0) {
+      int lv = 0;
+      if (!ptx::mbar_wait(kick, 0, limit, p.status)) limit = kWaitNsAfterFault;
+      for (int k = 0;; ++k) {
+        const int w = ring_item(k, item_full, ring, limit, p.status);
+        ptx::mbar_arrive(item_free + k % kRing);
+        if (w < 0) break;
         const AGeo g = attn_geo(p, w);
         if (!g.work) continue;
-        const int nk = g.nq - g.qt;
-        const int nv = p.a_out != nullptr && g.qt == 0 ? (g.NV + kTile - 1) / kTile : 0;
-        const int base_row = g.l * la.sum_T + g.t0;   // row of image position 0 in the maps
-        const int qb = it & 1;
-        if (it >= 2 && !ptx::mbar_wait(q_free + qb, ((it >> 1) - 1) & 1, limit, p.status))
-          limit = kWaitNsAfterFault;
-        ptx::mbar_arrive_expect_tx(q_full + qb, kTileBytes);
-        ptx::tma_load_3d(q_sm + qb * kTileBytes, &tmQ, q_full + qb, 0, g.h, base_row + g.row0);
-        ptx::tma_load_3d(q_sm + qb * kTileBytes + kHalfBytes, &tmQ, q_full + qb, 64, g.h,
-                         base_row + g.row0);
-        for (int jj = 0; jj < nk; ++jj) {
-          const int krow = base_row + g.T - kTile * (g.nq - jj);
-          load_k(krow, g.kvh);
-          const int s = lv & 1;
-          if (lv >= 2 && !ptx::mbar_wait(v_free + s, ((lv >> 1) - 1) & 1, limit, p.status))
+        const int base_row = g.l * la.sum_T + g.t0;
+        for (int j = 0; j < g.nq - g.qt; ++j) {
+          const int s = lv % kStages;
+          if (lv >= kStages && !ptx::mbar_wait(v_free + s, (lv / kStages - 1) & 1, limit, p.status))
             limit = kWaitNsAfterFault;
+          const int krow = base_row + g.T - kTile * (g.nq - j);
           ptx::mbar_arrive_expect_tx(v_full + s, kTileBytes);
           ptx::tma_load_3d(v_sm + s * kTileBytes, &tmV, v_full + s, 0, g.kvh, krow);
-          ptx::tma_load_3d(v_sm + s * kTileBytes + kHalfBytes, &tmV, v_full + s, 64, g.kvh,
-                           krow);
+          ptx::tma_load_3d(v_sm + s * kTileBytes + kHalfBytes, &tmV, v_full + s, 64, g.kvh, krow);
           ++lv;
         }
-        for (int vt = 0; vt < nv; ++vt) load_k(base_row + g.S + kTile * vt, g.kvh);
-        ++it;
       }
     }
-  } else if (warp == 1) {
-    // ================= MMA issuer
+  } else if (warp == kWarpQK) {
+    // ================= MMA: S = Q K^T for every key tile, then the score sweep
     if (lane == 0) {
       const uint32_t idesc_s = ptx::idesc_bf16_f32(kTile, kTile);
-      const uint32_t idesc_pv = ptx::idesc_bf16_f32(kTile, 128) | (1u << 16);   // B MN-major
-      int it = 0, sc = 0, pc = 0, lk = 0, lv = 0;
-      auto qk = [&](uint32_t b_base, uint32_t idesc, bool keys_on_lanes) {
-        const int sb = sc & 1;
-        if (sc >= 2 && !ptx::mbar_wait(s_free + sb, ((sc >> 1) - 1) & 1, limit, p.status))
-          limit = kWaitNsAfterFault;
-        const int s = lk & 1;
-        if (!ptx::mbar_wait(k_full + s, (lk >> 1) & 1, limit, p.status)) limit = kWaitNsAfterFault;
-        ptx::tc_fence_after();
-        const uint32_t k_base = ptx::smem_addr(k_sm + s * kTileBytes);
-#pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-          const uint32_t half = ks >> 2, kk = ks & 3;
-          const uint64_t qd = ptx::sdesc_sw128(b_base + half * kHalfBytes + kk * 32u);
-          const uint64_t kd = ptx::sdesc_sw128(k_base + half * kHalfBytes + kk * 32u);
-          ptx::mma_bf16(tmem + (uint32_t)sb * kColsS, keys_on_lanes ? kd : qd,
-                        keys_on_lanes ? qd : kd, idesc, ks > 0 ? 1u : 0u);
-        }
-        ptx::mma_commit(k_free + s);
-        ptx::mma_commit(s_full + sb);
-        ++sc;
-        ++lk;
-      };
-      auto pv = [&](bool first) {
-        const int pb = pc & 1;
-        if (!ptx::mbar_wait(p_ready + pb, (pc >> 1) & 1, limit, p.status)) limit = kWaitNsAfterFault;
-        const int s = lv & 1;
-        if (!ptx::mbar_wait(v_full + s, (lv >> 1) & 1, limit, p.status)) limit = kWaitNsAfterFault;
-        // the first P V of an item overwrites O: the previous item's O must be out
-        if (first && it >= 1 && !ptx::mbar_wait(o_free, (it - 1) & 1, limit, p.status))
-          limit = kWaitNsAfterFault;
-        ptx::tc_fence_after();
-        const uint32_t v_base = ptx::smem_addr(v_sm + s * kTileBytes);
-#pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-          const uint64_t vd = sdesc_sw128_mn(v_base + (uint32_t)ks * 2048u, (uint32_t)kHalfBytes);
-          mma_bf16_ts(tmem + kColO, tmem + kColP + (uint32_t)pb * 64u + (uint32_t)ks * 8u, vd,
-                      idesc_pv, (!first || ks > 0) ? 1u : 0u);
-        }
-        ptx::mma_commit(v_free + s);
-        ptx::mma_commit(pv_done + pb);
-        ++pc;
-        ++lv;
-      };
-      for (int kk = 0;; ++kk) {
-        const int w = attn_item(kk);
-        if (w >= p.items) break;
+      int it = 0, sc = 0, lk = 0;
+      for (int k = 0;; ++k) {
+        const int w = ring_item(k, item_full, ring, limit, p.status);
+        ptx::mbar_arrive(item_free + k % kRing);
+        if (w < 0) break;
         const AGeo g = attn_geo(p, w);
         if (!g.work) continue;
         const int nk = g.nq - g.qt;
-        const int nv = p.a_out != nullptr && g.qt == 0 ? (g.NV + kTile - 1) / kTile : 0;
-        const int ntp2 = max(16, (g.NT + 15) & ~15);   // text columns of the score sweep
-        const int qb = it & 1;
-        if (!ptx::mbar_wait(q_full + qb, (it >> 1) & 1, limit, p.status))
-          limit = kWaitNsAfterFault;
-        ptx::tc_fence_after();
-        const uint32_t q_base = ptx::smem_addr(q_sm + qb * kTileBytes);
-        for (int jj = 0; jj < nk; ++jj) {
-          qk(q_base, idesc_s, false);
-          if (jj >= 1) pv(jj == 1);
-        }
-        pv(nk == 1);
+        const int n = stream_ops(g, p, kOpsQK);
         // score sweep: D[key][t] = K_vis Q_text^T, the text rows (the last ntp2
         // rows of the tile, an 8-row-aligned start) as N
+        const int ntp2 = max(16, (g.NT + 15) & ~15);
         const uint32_t idesc_a = ptx::idesc_bf16_f32(kTile, ntp2);
-        for (int vt = 0; vt < nv; ++vt)
-          qk(q_base + (uint32_t)(kTile - ntp2) * 128u, idesc_a, true);
-        ptx::mma_commit(q_free + qb);
+        if (!ptx::mbar_wait(q_full, it & 1, limit, p.status)) limit = kWaitNsAfterFault;
+        for (int j = 0; j < n; ++j) {
+          const int sb = sc & 1, s = lk % kStages;
+          if (sc >= 2 && !ptx::mbar_wait(s_free + sb, ((sc >> 1) - 1) & 1, limit, p.status))
+            limit = kWaitNsAfterFault;
+          if (!ptx::mbar_wait(k_full + s, (lk / kStages) & 1, limit, p.status))
+            limit = kWaitNsAfterFault;
+          ptx::tc_fence_after();
+          const bool keys_on_lanes = j >= nk;
+          const uint32_t q_base = ptx::smem_addr(q_sm) +
+                                  (keys_on_lanes ? (uint32_t)(kTile - ntp2) * 128u : 0u);
+          const uint32_t idesc = keys_on_lanes ? idesc_a : idesc_s;
+          const uint32_t k_base = ptx::smem_addr(k_sm + s * kTileBytes);
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks) {
+            const uint32_t half = ks >> 2, k4 = ks & 3;
+            const uint64_t qd = ptx::sdesc_sw128(q_base + half * kHalfBytes + k4 * 32u);
+            const uint64_t kd = ptx::sdesc_sw128(k_base + half * kHalfBytes + k4 * 32u);
+            ptx::mma_bf16(tmem + (uint32_t)sb * kColsS, keys_on_lanes ? kd : qd,
+                          keys_on_lanes ? qd : kd, idesc, ks > 0 ? 1u : 0u);
+          }
+          ptx::mma_commit(k_free + s);
+          ptx::mma_commit(s_full + sb);
+          ++sc;
+          ++lk;
+        }
+        ptx::mma_commit(q_free);   // every MMA reading this item's Q is issued
+        ++it;
+      }
+      ptx::mma_commit(fin);
+      if (!ptx::mbar_wait(fin, 0, limit, p.status)) limit = kWaitNsAfterFault;
+    }
+  } else if (warp == kWarpPV) {
+    // ================= MMA: O += P V for every key tile
+    if (lane == 0) {
+      const uint32_t idesc_pv = ptx::idesc_bf16_f32(kTile, 128) | (1u << 16);   // B MN-major
+      int it = 0, pc = 0, lv = 0;
+      for (int k = 0;; ++k) {
+        const int w = ring_item(k, item_full, ring, limit, p.status);
+        ptx::mbar_arrive(item_free + k % kRing);
+        if (w < 0) break;
+        const AGeo g = attn_geo(p, w);
+        if (!g.work) continue;
+        for (int x = 0; x < g.nq - g.qt; ++x) {
+          const int pb = pc & 1, s = lv % kStages;
+          if (!ptx::mbar_wait(p_ready + pb, (pc >> 1) & 1, limit, p.status))
+            limit = kWaitNsAfterFault;
+          if (!ptx::mbar_wait(v_full + s, (lv / kStages) & 1, limit, p.status))
+            limit = kWaitNsAfterFault;
+          // the first P V of an item overwrites O: the previous item's O must be out
+          if (x == 0 && it >= 1 && !ptx::mbar_wait(o_free, (it - 1) & 1, limit, p.status))
+            limit = kWaitNsAfterFault;
+          ptx::tc_fence_after();
+          const uint32_t v_base = ptx::smem_addr(v_sm + s * kTileBytes);
+#pragma unroll
+          for (int ks = 0; ks < 8; ++ks) {
+            const uint64_t vd = sdesc_sw128_mn(v_base + (uint32_t)ks * 2048u, (uint32_t)kHalfBytes);
+            mma_bf16_ts(tmem + kColO, tmem + kColP + (uint32_t)pb * 64u + (uint32_t)ks * 8u, vd,
+                        idesc_pv, (x > 0 || ks > 0) ? 1u : 0u);
+          }
+          ptx::mma_commit(v_free + s);
+          ptx::mma_commit(pv_done + pb);
+          ++pc;
+          ++lv;
+        }
         ++it;
       }
       ptx::mma_commit(fin);
@@ -430,9 +526,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_base = (uint32_t)(q4 * 32) << 16;
     const uint32_t pair_bar = 2u + (uint32_t)q4;   // the two warps of this lane quarter
     int it = 0, sc = 0, pc = 0;
-    for (int kk = 0;; ++kk) {
-      const int w = attn_item(kk);
-      if (w >= p.items) break;
+    for (int k = 0;; ++k) {
+      // one thread takes the item from the ring for all eight warps, so they
+      // always agree (their named barriers depend on it)
+      if (threadIdx.x == 64) {
+        sm_item[k & 1] = ring_item(k, item_full, ring, limit, p.status);
+        ptx::mbar_arrive(item_free + k % kRing);
+      }
+      ptx::named_bar(1, kEpiThreads);
+      const int w = sm_item[k & 1];
+      if (w < 0) break;
       const AGeo g = attn_geo(p, w);
       if (!g.ok && g.qt == 0 && threadIdx.x == 64) E2S_DEV_FLAG(p.status, E2S_ERR_SHAPE);
       if (!g.work) continue;
@@ -472,10 +575,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 16; i < 64; ++i) mx[i & 7] = fmaxf(mx[i & 7], s[i]);
         const float hmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
                                  fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
-        float* xb = xch + (pc & 1) * 2 * kTile;
-        xb[ch * kTile + r] = hmax;
+        xch[ch * kTile + r] = hmax;
         ptx::named_bar(pair_bar, 64);
-        const float tmax = fmaxf(xb[r], xb[kTile + r]);
+        const float tmax = fmaxf(xch[r], xch[kTile + r]);
+        ptx::named_bar(pair_bar, 64);   // xch is rewritten only after both halves read it
         const float tm = tmax > 0.5f * kNegBig ? tmax * p.scale_log2 : kNegBig;
         // the reference maximum moves only by more than kLazy (or from empty)
         const bool move = tm > m + kLazy || (m <= 0.5f * kNegBig && tm > 0.5f * kNegBig);
@@ -522,10 +625,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) ptx::mbar_arrive(p_ready + pb);
         ++pc;
       }
-      // ---- O / l and the row normaliser (the two halves' sums meet in xsum)
-      xsum[ch * kTile + r] = lsum;
+      // ---- O / l and the row normaliser (the two halves' sums meet in xch)
+      xch[ch * kTile + r] = lsum;
       ptx::named_bar(pair_bar, 64);
-      const float ltot = xsum[r] + xsum[kTile + r];
+      const float ltot = xch[r] + xch[kTile + r];
+      ptx::named_bar(pair_bar, 64);   // xch is rewritten only after both halves read it
       {
         const int pl = (pc - 1) & 1;
         if (!ptx::mbar_wait(pv_done + pl, ((pc - 1) >> 1) & 1, limit, p.status))
@@ -540,8 +644,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) ptx::mbar_arrive(o_free);   // the next item's P V may overwrite O
       if (rvalid) {
         const float inv = ltot > 0.f ? 1.f / ltot : 0.f;
-        uint4* orow = reinterpret_cast<uint4*>(
-            p.o_out + (int64_t)(base_row + qp) * p.o_stride + (int64_t)g.h * 128 + c0);
+        uint16_t* orow16 = p.o_out + (int64_t)(base_row + qp) * p.o_stride + (int64_t)g.h * 128 + c0;
+        uint4* orow = reinterpret_cast<uint4*>(orow16);
+        if (p.o_v8) {
+          // a row's 128 bytes in four 32-byte stores (each store instruction of
+          // the warp touches 32 rows, so wider stores mean fewer transactions)
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            const float* o = j == 0 ? o0 : o1;
+#pragma unroll
+            for (int h2 = 0; h2 < 2; ++h2) {
+              const float* x = o + 16 * h2;
+              st_global_v8(orow16 + 32 * j + 16 * h2, pack_bf16(x[0] * inv, x[1] * inv),
+                           pack_bf16(x[2] * inv, x[3] * inv), pack_bf16(x[4] * inv, x[5] * inv),
+                           pack_bf16(x[6] * inv, x[7] * inv), pack_bf16(x[8] * inv, x[9] * inv),
+                           pack_bf16(x[10] * inv, x[11] * inv),
+                           pack_bf16(x[12] * inv, x[13] * inv),
+                           pack_bf16(x[14] * inv, x[15] * inv));
+            }
+          }
+        } else {
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           orow[j] = make_uint4(pack_bf16(o0[8 * j] * inv, o0[8 * j + 1] * inv),
@@ -552,6 +674,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                    pack_bf16(o1[8 * j + 2] * inv, o1[8 * j + 3] * inv),
                                    pack_bf16(o1[8 * j + 4] * inv, o1[8 * j + 5] * inv),
                                    pack_bf16(o1[8 * j + 6] * inv, o1[8 * j + 7] * inv));
+        }
         }
       }
       const float lse2 = ltot > 0.f ? m + __log2f(ltot) : -kNegBig;
@@ -564,7 +687,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---- the score from the final row normalisers: keys on the lanes,
         // column c <-> tile row kTile - ntp2 + c <-> text row c - (ntp2 - NT);
         // the two warps of a lane quarter take alternate 16-column chunks
-        ptx::named_bar(1, kEpiThreads);   // nlse complete, xsum read by every warp
+        ptx::named_bar(1, kEpiThreads);   // nlse complete
         const int c_text = ntp2 - g.NT;
         const float inv_nt = 1.f / (float)g.NT;
         float st_s = 0.f, st_m = kNegBig, st_e = 0.f;
@@ -586,18 +709,18 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) ptx::mbar_arrive(s_free + sb);
           ++sc;
-          xsum[ch * kTile + r] = acc;
+          xch[ch * kTile + r] = acc;
           ptx::named_bar(pair_bar, 64);
           const int key = kTile * vt + r;   // visual index of this lane's key
           if (ch == 0 && key < g.NV) {
-            const float a = (xsum[r] + xsum[kTile + r]) * inv_nt;
+            const float a = (xch[r] + xch[kTile + r]) * inv_nt;
             p.a_out[((size_t)g.l * la.H + g.h) * (size_t)la.sum_vis + g.v0 + key] = a;
             const float al = a * kLog2e, mn = fmaxf(st_m, al);
             st_e = st_e * fast_ex2(st_m - mn) + fast_ex2(al - mn);
             st_m = mn;
             st_s += a;
           }
-          ptx::named_bar(pair_bar, 64);   // xsum is rewritten by the next tile
+          ptx::named_bar(pair_bar, 64);   // xch is rewritten by the next tile
         }
         if (ch == 0) {
 #pragma unroll
@@ -626,9 +749,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   ptx::tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
+  if (warp == kWarpQK) {
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, 512);
+  }
+  if (threadIdx.x == 0) {
+    // the last CTA out (every CTA has taken its last item) zeroes the counter
+    __threadfence();
+    if (atomicAdd(p.sched + 1, 1u) == gridDim.x - 1) {
+      atomicExch(p.sched, 0u);
+      atomicExch(p.sched + 1, 0u);
+    }
   }
 }
 
@@ -637,7 +768,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 cudaError_t launch_attention(const LayoutArgs& la, const void* q, int64_t q_stride, const void* k,
                              int64_t k_stride, const void* v, int64_t v_stride, void* o_out,
                              int64_t o_stride, float* lse_out, float* a_out, float4* stats,
-                             uint32_t* counters, uint32_t* status, cudaStream_t st) {
+                             uint32_t* counters, uint32_t* sched, uint32_t* status,
+                             cudaStream_t st) {
   AttnArgs p;
   p.la = la;
   p.group = la.H / la.H_kv;
@@ -645,10 +777,12 @@ cudaError_t launch_attention(const LayoutArgs& la, const void* q, int64_t q_stri
   p.scale_log2 = 1.4426950408889634f / sqrtf(128.0f);
   p.o_out = static_cast<uint16_t*>(o_out);
   p.o_stride = o_stride;
+  p.o_v8 = (reinterpret_cast<uintptr_t>(o_out) % 32 == 0 && o_stride % 16 == 0) ? 1 : 0;
   p.lse_out = lse_out;
   p.a_out = a_out;
   p.stats = stats;
   p.counters = counters;
+  p.sched = sched;
   p.status = status;
   if (p.units == 0 || la.max_T == 0) return cudaSuccess;
   const int n_qt = (la.max_T + kTile - 1) / kTile;

@@ -264,7 +264,8 @@ e2s_status e2s_attention(const e2s_layout* layout, const void* q, int64_t q_row_
   return from_cuda(launch_attention(layout_args(layout), q, q_row_stride, k, k_row_stride, v,
                                     v_row_stride, o_out, o_row_stride, lse_out, a_out,
                                     stats_ptr(ws), a_out ? decide_scratch_ptr(ws, layout) : nullptr,
-                                    status_word(ws), static_cast<cudaStream_t>(stream)));
+                                    attn_sched_ptr(ws), status_word(ws),
+                                    static_cast<cudaStream_t>(stream)));
 }
 
 e2s_status e2s_decide_attn(const e2s_layout* layout, const e2s_params* params, const void* q,
@@ -454,7 +455,7 @@ e2s_status e2s_read_status(const void* ws, void* stream) {
 
 e2s_status e2s_clear_status(void* ws, void* stream) {
   if (!ws) return E2S_ERR_WORKSPACE;
-  return from_cuda(cudaMemsetAsync(ws, 0, sizeof(uint32_t), static_cast<cudaStream_t>(stream)));
+  return from_cuda(cudaMemsetAsync(ws, 0, kClearBytes, static_cast<cudaStream_t>(stream)));
 }
 
 const char* e2s_status_string(e2s_status s) {

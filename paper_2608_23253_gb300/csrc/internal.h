@@ -8,7 +8,8 @@
 
 namespace e2s {
 
-// Workspace layout: [0, 256) status word + reserved; then one float4 of
+// Workspace layout: [0, 256) status word, attention item counter and
+// finished-CTA count (words 1 and 2), reserved; then one float4 of
 // normalisation statistics per (image, layer, head) -- (S, M, 1/E, 1/S) with
 // S = sum of a, M = max of a*log2e, E = sum of 2^(a*log2e - M) over the image's
 // visual tokens (stats_entry), written by the score kernels; then the decision scratch of e2s_decide: per image 64
@@ -25,6 +26,10 @@ inline size_t decide_scratch_bytes(const e2s_layout* L) {
   return ((size_t)L->B * kDecideWordsPerImage * sizeof(uint32_t) + 255) & ~(size_t)255;
 }
 inline uint32_t* status_word(void* ws) { return reinterpret_cast<uint32_t*>(ws); }
+// Words 1 and 2 of the status area: the attention kernel's shared item counter
+// and its count of finished CTAs (zero between calls).
+inline uint32_t* attn_sched_ptr(void* ws) { return reinterpret_cast<uint32_t*>(ws) + 1; }
+constexpr size_t kClearBytes = 16;   // bytes of the status area zeroed before first use
 inline float4* stats_ptr(void* ws) {
   return reinterpret_cast<float4*>(reinterpret_cast<char*>(ws) + kStatusBytes);
 }
@@ -87,10 +92,13 @@ cudaError_t launch_score_split(const LayoutArgs& la, int mode, const void* q, in
                                const float* lse_in, int cluster, int tpc);
 // The pruning layer's causal attention (O and the row lse) with the text rows'
 // score a and its Eq. 8 statistics as a by-product when a_out is given.
+// sched: two workspace words, zero on entry and on return (the item counter
+// the CTAs share).
 cudaError_t launch_attention(const LayoutArgs& la, const void* q, int64_t q_stride, const void* k,
                              int64_t k_stride, const void* v, int64_t v_stride, void* o_out,
                              int64_t o_stride, float* lse_out, float* a_out, float4* stats,
-                             uint32_t* counters, uint32_t* status, cudaStream_t st);
+                             uint32_t* counters, uint32_t* sched, uint32_t* status,
+                             cudaStream_t st);
 // Persistent single-CTA-per-unit score kernel and its applicability tests.
 bool score_unit_fits(const LayoutArgs& la, int mode);
 bool score_unit_single_group(const LayoutArgs& la, int mode);

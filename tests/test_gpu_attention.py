@@ -109,3 +109,61 @@ def test_attention_score_equals_separate_score():
     dec.score(bf16_tensor(inp.q_text, device()), bf16_tensor(inp.k, device()))
     torch.cuda.synchronize()
     parity.check_a(a_attn, dec.a.cpu().numpy().astype(np.float64), causal=True, rel=1e-5)
+
+
+def _attention_raw(inp, dec, q, k, v, o, o_stride, lse):
+    from paper_2608_23253_gb300 import e2s
+    b = dec.batch
+    e2s.check(e2s.e2s_attention(b.layout, q, b.H * b.d, k, b.H_kv * b.d, v, b.H_kv * b.d, o,
+                                o_stride, lse, dec.a, dec.ws, dec.ws_bytes, None),
+              "e2s_attention")
+
+
+def test_attention_unaligned_output_rows():
+    """O rows that are 16- but not 32-byte aligned (offset 16 bytes, row stride
+    H*d + 8) take the 16-byte store path: the same bits as the aligned run, and
+    the padding between rows untouched."""
+    from paper_2608_23253_gb300 import e2s
+    from paper_2608_23253_gb300.decision import Batch, Decision, bf16_tensor
+    inp = _cases("gqa-ragged")
+    _, dec, o_ref, lse_ref = _run(inp)
+    dev = device()
+    s = inp.spec
+    q = bf16_tensor(synth.full_queries(inp), dev)
+    k, v = bf16_tensor(inp.k, dev), bf16_tensor(inp.v, dev)
+    rows, width = s.L * dec.batch.sum_T, s.H * 128
+    big = torch.full((rows, width + 8), 7.0, dtype=torch.bfloat16, device=dev)
+    o = big[:, 8:8 + width]
+    assert o.data_ptr() % 32 == 16
+    lse = torch.full((s.L, s.H, dec.batch.sum_T), float("nan"), dtype=torch.float32, device=dev)
+    _attention_raw(inp, dec, q, k, v, o, width + 8, lse)
+    torch.cuda.synchronize()
+    assert dec.status() == e2s.E2S_OK
+    got = o.float().cpu().numpy().reshape(o_ref.shape)
+    assert np.array_equal(got.view(np.uint32), o_ref.view(np.uint32))
+    assert np.array_equal(lse.cpu().numpy(), lse_ref)
+    assert bool((big[:, :8] == 7.0).all())
+
+
+def test_attention_repeats_and_leaves_counter_zero():
+    """The CTAs share an item counter in the workspace: 50 calls in a row give
+    the same bits every time and leave workspace bytes 4..15 zero."""
+    from paper_2608_23253_gb300 import e2s
+    from paper_2608_23253_gb300.decision import bf16_tensor
+    inp = _cases("cfg0")
+    _, dec, o_ref, lse_ref = _run(inp)
+    dev = device()
+    s = inp.spec
+    q = bf16_tensor(synth.full_queries(inp), dev)
+    k, v = bf16_tensor(inp.k, dev), bf16_tensor(inp.v, dev)
+    o = torch.empty_like(q)
+    lse = torch.empty((s.L, s.H, dec.batch.sum_T), dtype=torch.float32, device=dev)
+    a_ref = dec.a.clone()
+    for _ in range(50):
+        dec.attention(q, k, v, o, lse)
+    torch.cuda.synchronize()
+    assert dec.status() == e2s.E2S_OK
+    assert np.array_equal(o.float().cpu().numpy().view(np.uint32), o_ref.view(np.uint32))
+    assert np.array_equal(lse.cpu().numpy(), lse_ref)
+    assert torch.equal(dec.a, a_ref)
+    assert int(dec.ws[4:16].to(torch.int32).abs().sum()) == 0
