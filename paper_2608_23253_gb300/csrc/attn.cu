@@ -81,7 +81,6 @@ struct AttnArgs {
   float scale_log2;     // log2(e) / sqrt(d)
   uint16_t* o_out;      // [L][sum_T] rows of (H x d) bf16
   int64_t o_stride;     // elements between consecutive rows
-  int o_v8;             // o_out and its rows are 32-byte aligned: 32-byte stores
   float* lse_out;       // nullable [L][H][sum_T]
   float* a_out;         // nullable [L][H][sum_vis]
   float4* stats;        // per (image, layer, head), written with a_out
@@ -105,8 +104,8 @@ __host__ __device__ inline APlan attn_plan() {
   s.k = kTileBytes;
   s.v = s.k + kStages * kTileBytes;
   s.bars = s.v + kStages * kTileBytes;
-  s.slot = s.bars + 8u * kBars;           // TMEM address, softmax item [2], item ring [kRing]
-  s.nlse = (s.slot + 32u + 15u) & ~15u;   // float [128]
+  s.slot = s.bars + 8u * kBars;           // TMEM address, softmax flags [2], ring [kRing][8]
+  s.nlse = (s.slot + 16u + 32u * kRing + 15u) & ~15u;   // float [128]
   s.xch = s.nlse + kTile * 4u;            // float [2][128]: the two column halves of a row
   s.red = s.xch + 2 * kTile * 4u;         // float4 [4]
   s.total = s.red + 4 * 16u;
@@ -132,14 +131,6 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 
 __device__ __forceinline__ float neg_inf() { return __int_as_float(0xff800000); }
 
-// 32-byte global store (8 packed words).
-__device__ __forceinline__ void st_global_v8(void* p, uint32_t a0, uint32_t a1, uint32_t a2,
-                                             uint32_t a3, uint32_t a4, uint32_t a5, uint32_t a6,
-                                             uint32_t a7) {
-  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(a0),
-               "r"(a1), "r"(a2), "r"(a3), "r"(a4), "r"(a5), "r"(a6), "r"(a7)
-               : "memory");
-}
 
 // D (TMEM) (+)= A B with A read from TMEM (row i of A on lane i; for 16-bit
 // types two consecutive K elements per 32-bit column, the lower index in the
@@ -252,16 +243,49 @@ __device__ __forceinline__ AGeo attn_geo(const AttnArgs& p, int w) {
   return g;
 }
 
-// Item k of this CTA's walk, as the K-load warp published it in the ring
-// (-1: no more items, or the wait ran out).
-__device__ __forceinline__ int ring_item(int k, uint64_t* item_full, const volatile int* ring,
-                                         uint64_t& limit, uint32_t* status) {
-  const int slot = k % kRing;
-  if (!ptx::mbar_wait(item_full + slot, (k / kRing) & 1, limit, status)) {
-    limit = kWaitNsAfterFault;
-    return -1;
-  }
-  return ring[slot];
+// A ring entry: the item index (-1: no more items) and its image's geometry,
+// so that only the K-load warp reads the layout arrays.
+constexpr int kRingInts = 8;
+
+__device__ __forceinline__ void ring_put(volatile int* e, int w, const AGeo& g) {
+  e[0] = w;
+  e[1] = g.S;
+  e[2] = g.NV;
+  e[3] = g.NT;
+  e[4] = g.t0;
+  e[5] = g.v0;
+  e[6] = g.ok ? 1 : 0;
+}
+
+__device__ __forceinline__ AGeo ring_geo(const volatile int* e, const AttnArgs& p) {
+  const LayoutArgs& la = p.la;
+  AGeo g;
+  const int w = e[0];
+  const int unit = w % p.units;
+  g.qt = w / p.units;
+  g.h = unit % la.H;
+  g.l = (unit / la.H) % la.L;
+  g.b = unit / (la.H * la.L);
+  g.kvh = g.h / p.group;
+  g.S = e[1];
+  g.NV = e[2];
+  g.NT = e[3];
+  g.t0 = e[4];
+  g.v0 = e[5];
+  g.ok = e[6] != 0;
+  g.T = g.S + g.NV + g.NT;
+  g.nq = g.ok ? (g.T + kTile - 1) / kTile : 0;
+  g.row0 = g.T - kTile * (g.qt + 1);
+  g.work = g.qt < g.nq;
+  return g;
+}
+
+// Waits for ring slot k (false: the wait ran out).
+__device__ __forceinline__ bool ring_wait(int k, uint64_t* item_full, uint64_t& limit,
+                                          uint32_t* status) {
+  if (ptx::mbar_wait(item_full + k % kRing, (k / kRing) & 1, limit, status)) return true;
+  limit = kWaitNsAfterFault;
+  return false;
 }
 
 // Per item: nk + nv key tiles and S tiles (nv visual key tiles of the score
@@ -301,7 +325,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* item_free = item_full + kRing;   // [kRing] ring slot read by every role
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + plan.slot);
   volatile int* sm_item = reinterpret_cast<volatile int*>(smem + plan.slot + 4);    // [2]
-  volatile int* ring = reinterpret_cast<volatile int*>(smem + plan.slot + 16);      // [kRing]
+  volatile int* ring = reinterpret_cast<volatile int*>(smem + plan.slot + 16);      // [kRing][8]
   float* nlse = reinterpret_cast<float*>(smem + plan.nlse);
   float* xch = reinterpret_cast<float*>(smem + plan.xch);
   float4* red = reinterpret_cast<float4*>(smem + plan.red);
@@ -361,15 +385,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int slot = k % kRing;
         if (k >= kRing && !ptx::mbar_wait(item_free + slot, (k / kRing - 1) & 1, limit, p.status))
           limit = kWaitNsAfterFault;
-        ring[slot] = w < p.items ? w : -1;
+        volatile int* e = ring + slot * kRingInts;
+        if (w < p.items) {
+          const AGeo g = attn_geo(p, w);
+          if (!g.ok && g.qt == 0) E2S_DEV_FLAG(p.status, E2S_ERR_SHAPE);
+          ring_put(e, w, g);
+        } else {
+          e[0] = -1;
+        }
         ptx::mbar_arrive(item_full + slot);
       };
       publish(0, (int)blockIdx.x);
       for (int k = 0;; ++k) {
-        const int w = ring[k % kRing];
-        if (w < 0) break;
+        const volatile int* e = ring + (k % kRing) * kRingInts;
+        if (e[0] < 0) break;
         const uint32_t nxt = atomicAdd(p.sched, 1u);   // published after this item's loads
-        const AGeo g = attn_geo(p, w);
+        const AGeo g = ring_geo(e, p);
         if (g.work) {
         const int nk = g.nq - g.qt;
         const int n = stream_ops(g, p, kOpsQK);
@@ -411,10 +442,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       int lv = 0;
       if (!ptx::mbar_wait(kick, 0, limit, p.status)) limit = kWaitNsAfterFault;
       for (int k = 0;; ++k) {
-        const int w = ring_item(k, item_full, ring, limit, p.status);
+        const volatile int* e = ring + (k % kRing) * kRingInts;
+        const bool more = ring_wait(k, item_full, limit, p.status) && e[0] >= 0;
+        const AGeo g = ring_geo(e, p);
         ptx::mbar_arrive(item_free + k % kRing);
-        if (w < 0) break;
-        const AGeo g = attn_geo(p, w);
+        if (!more) break;
         if (!g.work) continue;
         const int base_row = g.l * la.sum_T + g.t0;
         for (int j = 0; j < g.nq - g.qt; ++j) {
@@ -435,10 +467,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t idesc_s = ptx::idesc_bf16_f32(kTile, kTile);
       int it = 0, sc = 0, lk = 0;
       for (int k = 0;; ++k) {
-        const int w = ring_item(k, item_full, ring, limit, p.status);
+        const volatile int* e = ring + (k % kRing) * kRingInts;
+        const bool more = ring_wait(k, item_full, limit, p.status) && e[0] >= 0;
+        const AGeo g = ring_geo(e, p);
         ptx::mbar_arrive(item_free + k % kRing);
-        if (w < 0) break;
-        const AGeo g = attn_geo(p, w);
+        if (!more) break;
         if (!g.work) continue;
         const int nk = g.nq - g.qt;
         const int n = stream_ops(g, p, kOpsQK);
@@ -484,10 +517,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t idesc_pv = ptx::idesc_bf16_f32(kTile, 128) | (1u << 16);   // B MN-major
       int it = 0, pc = 0, lv = 0;
       for (int k = 0;; ++k) {
-        const int w = ring_item(k, item_full, ring, limit, p.status);
+        const volatile int* e = ring + (k % kRing) * kRingInts;
+        const bool more = ring_wait(k, item_full, limit, p.status) && e[0] >= 0;
+        const AGeo g = ring_geo(e, p);
         ptx::mbar_arrive(item_free + k % kRing);
-        if (w < 0) break;
-        const AGeo g = attn_geo(p, w);
+        if (!more) break;
         if (!g.work) continue;
         for (int x = 0; x < g.nq - g.qt; ++x) {
           const int pb = pc & 1, s = lv % kStages;
@@ -529,15 +563,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int k = 0;; ++k) {
       // one thread takes the item from the ring for all eight warps, so they
       // always agree (their named barriers depend on it)
-      if (threadIdx.x == 64) {
-        sm_item[k & 1] = ring_item(k, item_full, ring, limit, p.status);
-        ptx::mbar_arrive(item_free + k % kRing);
-      }
+      if (threadIdx.x == 64) sm_item[k & 1] = ring_wait(k, item_full, limit, p.status) ? 1 : 0;
       ptx::named_bar(1, kEpiThreads);
-      const int w = sm_item[k & 1];
-      if (w < 0) break;
-      const AGeo g = attn_geo(p, w);
-      if (!g.ok && g.qt == 0 && threadIdx.x == 64) E2S_DEV_FLAG(p.status, E2S_ERR_SHAPE);
+      // every softmax warp has read entry k - 1 (it reached this barrier)
+      if (threadIdx.x == 64 && k >= 1) ptx::mbar_arrive(item_free + (k - 1) % kRing);
+      const volatile int* e = ring + (k % kRing) * kRingInts;
+      if (sm_item[k & 1] == 0 || e[0] < 0) break;
+      const AGeo g = ring_geo(e, p);
       if (!g.work) continue;
       const int nk = g.nq - g.qt;
       const bool sweep = p.a_out != nullptr && g.qt == 0 && g.NV > 0;
@@ -642,39 +674,44 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::tc_fence_before();
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(o_free);   // the next item's P V may overwrite O
-      if (rvalid) {
+      {
+        // O / l in bf16: the lane's 128 bytes of its row as eight 16-byte
+        // chunks, transposed within each group of 8 lanes (three butterfly
+        // exchanges) so that lane 8 g + i then holds chunk i of the group's 8
+        // rows; each store instruction of the warp then writes 4 whole rows
         const float inv = ltot > 0.f ? 1.f / ltot : 0.f;
-        uint16_t* orow16 = p.o_out + (int64_t)(base_row + qp) * p.o_stride + (int64_t)g.h * 128 + c0;
-        uint4* orow = reinterpret_cast<uint4*>(orow16);
-        if (p.o_v8) {
-          // a row's 128 bytes in four 32-byte stores (each store instruction of
-          // the warp touches 32 rows, so wider stores mean fewer transactions)
+        uint32_t wd[32];
 #pragma unroll
-          for (int j = 0; j < 2; ++j) {
-            const float* o = j == 0 ? o0 : o1;
+        for (int j2 = 0; j2 < 16; ++j2) {
+          wd[j2] = pack_bf16(o0[2 * j2] * inv, o0[2 * j2 + 1] * inv);
+          wd[16 + j2] = pack_bf16(o1[2 * j2] * inv, o1[2 * j2 + 1] * inv);
+        }
 #pragma unroll
-            for (int h2 = 0; h2 < 2; ++h2) {
-              const float* x = o + 16 * h2;
-              st_global_v8(orow16 + 32 * j + 16 * h2, pack_bf16(x[0] * inv, x[1] * inv),
-                           pack_bf16(x[2] * inv, x[3] * inv), pack_bf16(x[4] * inv, x[5] * inv),
-                           pack_bf16(x[6] * inv, x[7] * inv), pack_bf16(x[8] * inv, x[9] * inv),
-                           pack_bf16(x[10] * inv, x[11] * inv),
-                           pack_bf16(x[12] * inv, x[13] * inv),
-                           pack_bf16(x[14] * inv, x[15] * inv));
+        for (int d = 4; d >= 1; d >>= 1) {
+          const bool upper = (lane & d) != 0;
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            if ((c & d) != 0) continue;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const uint32_t send = upper ? wd[4 * c + q] : wd[4 * (c | d) + q];
+              const uint32_t recv = __shfl_xor_sync(0xffffffffu, send, d);
+              if (upper) {
+                wd[4 * c + q] = recv;
+              } else {
+                wd[4 * (c | d) + q] = recv;
+              }
             }
           }
-        } else {
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          orow[j] = make_uint4(pack_bf16(o0[8 * j] * inv, o0[8 * j + 1] * inv),
-                               pack_bf16(o0[8 * j + 2] * inv, o0[8 * j + 3] * inv),
-                               pack_bf16(o0[8 * j + 4] * inv, o0[8 * j + 5] * inv),
-                               pack_bf16(o0[8 * j + 6] * inv, o0[8 * j + 7] * inv));
-          orow[4 + j] = make_uint4(pack_bf16(o1[8 * j] * inv, o1[8 * j + 1] * inv),
-                                   pack_bf16(o1[8 * j + 2] * inv, o1[8 * j + 3] * inv),
-                                   pack_bf16(o1[8 * j + 4] * inv, o1[8 * j + 5] * inv),
-                                   pack_bf16(o1[8 * j + 6] * inv, o1[8 * j + 7] * inv));
         }
+        const int grow = q4 * 32 + (lane & ~7);   // tile row of the lane group's first row
+        uint16_t* obase = p.o_out + (int64_t)g.h * 128 + c0 + 8 * (lane & 7);
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const int qc = g.row0 + grow + c;        // image position of row grow + c
+          if (qc >= 0)
+            *reinterpret_cast<uint4*>(obase + (int64_t)(base_row + qc) * p.o_stride) =
+                make_uint4(wd[4 * c], wd[4 * c + 1], wd[4 * c + 2], wd[4 * c + 3]);
         }
       }
       const float lse2 = ltot > 0.f ? m + __log2f(ltot) : -kNegBig;
@@ -777,7 +814,6 @@ cudaError_t launch_attention(const LayoutArgs& la, const void* q, int64_t q_stri
   p.scale_log2 = 1.4426950408889634f / sqrtf(128.0f);
   p.o_out = static_cast<uint16_t*>(o_out);
   p.o_stride = o_stride;
-  p.o_v8 = (reinterpret_cast<uintptr_t>(o_out) % 32 == 0 && o_stride % 16 == 0) ? 1 : 0;
   p.lse_out = lse_out;
   p.a_out = a_out;
   p.stats = stats;
