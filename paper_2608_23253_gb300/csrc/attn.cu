@@ -337,7 +337,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
       p.counters[i] = 0u;
 
-  if (warp == 0 && lane == 0) {
+  uint64_t limit = kWaitNs;
+  int pk_lk = 0, pk_j0 = 0;   // K-load warp: key tiles already issued, first j of item 0
+  if (warp == kWarpLoadK && lane == 0) {
+    ptx::prefetch_tensormap(&tmQ);
+    ptx::prefetch_tensormap(&tmK);
+    ptx::prefetch_tensormap(&tmV);
     ptx::mbar_init(q_full, 1);
     ptx::mbar_init(q_free, 1);
     for (int i = 0; i < kStages; ++i) {
@@ -361,13 +366,31 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     ptx::fence_barrier_init();
     ptx::fence_proxy_async_smem();
+    // item 0 and, when it has work, its Q and first key tile go out before the
+    // block-wide setup barrier: these loads are the first S's critical path
+    const int w0 = (int)blockIdx.x;   // < items (the grid is at most the item count)
+    const AGeo g0 = attn_geo(p, w0);
+    if (!g0.ok && g0.qt == 0) E2S_DEV_FLAG(p.status, E2S_ERR_SHAPE);
+    ring_put(ring, w0, g0);
+    ptx::mbar_arrive(item_full);
+    if (g0.work) {
+      const int base_row = g0.l * la.sum_T + g0.t0;
+      const int krow = base_row + g0.T - kTile * g0.nq;
+      ptx::mbar_arrive_expect_tx(q_full, kTileBytes);
+      ptx::tma_load_3d(q_sm, &tmQ, q_full, 0, g0.h, base_row + g0.row0);
+      ptx::tma_load_3d(q_sm + kHalfBytes, &tmQ, q_full, 64, g0.h, base_row + g0.row0);
+      ptx::mbar_arrive_expect_tx(k_full, kTileBytes);
+      ptx::tma_load_3d(k_sm, &tmK, k_full, 0, g0.kvh, krow);
+      ptx::tma_load_3d(k_sm + kHalfBytes, &tmK, k_full, 64, g0.kvh, krow);
+      pk_lk = 1;
+      pk_j0 = 1;
+    }
   }
   if (warp == kWarpQK) ptx::tmem_alloc(tmem_slot, 512);
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  uint64_t limit = kWaitNs;
 
   if (warp == kWarpLoadK) {
     // ================= the item walk and TMA of each item's key tiles (then
@@ -375,12 +398,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     // previous item's last S = Q K^T is complete (after the item's first two
     // key tiles).  A CTA's first item is its block index; the next ones come
     // from one counter shared by all CTAs, in item order (the heaviest query
-    // tiles first), one item ahead, through the ring.  The first item's Q and
-    // first key tile go out alone, so that the first S is not queued behind
-    // every other load of the start.
+    // tiles first), through the ring.  The first item's Q and first key tile
+    // go out alone (before the setup barrier), so that the first S is not
+    // queued behind every other load of the start.
     if (lane == 0) {
-      int it = 0, lk = 0;
+      int it = 0, lk = pk_lk;
       bool kicked = false;
+      // the first value tile and the next key tiles wait for the first Q and
+      // key tile (only this thread completes these phases: the waits cannot alias)
+      auto kick_once = [&]() {
+        if (kicked || lk == 0) return;
+        if (!ptx::mbar_wait(q_full, 0, limit, p.status)) limit = kWaitNsAfterFault;
+        if (!ptx::mbar_wait(k_full, 0, limit, p.status)) limit = kWaitNsAfterFault;
+        ptx::mbar_arrive(kick);
+        kicked = true;
+      };
       auto publish = [&](int k, int w) {
         const int slot = k % kRing;
         if (k >= kRing && !ptx::mbar_wait(item_free + slot, (k / kRing - 1) & 1, limit, p.status))
@@ -395,17 +427,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         ptx::mbar_arrive(item_full + slot);
       };
-      publish(0, (int)blockIdx.x);
       for (int k = 0;; ++k) {
         const volatile int* e = ring + (k % kRing) * kRingInts;
         if (e[0] < 0) break;
-        const uint32_t nxt = atomicAdd(p.sched, 1u);   // published after this item's loads
         const AGeo g = ring_geo(e, p);
         if (g.work) {
         const int nk = g.nq - g.qt;
         const int n = stream_ops(g, p, kOpsQK);
         const int base_row = g.l * la.sum_T + g.t0;   // row of image position 0 in the maps
-        for (int j = 0; j < n; ++j) {
+        for (int j = k == 0 ? pk_j0 : 0; j < n; ++j) {
+          kick_once();
           if (it == 0 ? j == 0 : j == min(2, n - 1)) {
             if (it >= 1 && !ptx::mbar_wait(q_free, (it - 1) & 1, limit, p.status))
               limit = kWaitNsAfterFault;
@@ -422,17 +453,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           ptx::tma_load_3d(k_sm + s * kTileBytes, &tmK, k_full + s, 0, g.kvh, krow);
           ptx::tma_load_3d(k_sm + s * kTileBytes + kHalfBytes, &tmK, k_full + s, 64, g.kvh, krow);
           ++lk;
-          if (!kicked) {
-            // only this thread completes these phases, so the waits cannot alias
-            if (!ptx::mbar_wait(q_full, 0, limit, p.status)) limit = kWaitNsAfterFault;
-            if (!ptx::mbar_wait(k_full, 0, limit, p.status)) limit = kWaitNsAfterFault;
-            ptx::mbar_arrive(kick);
-            kicked = true;
-          }
         }
+        kick_once();
         ++it;
         }
-        publish(k + 1, (int)(gridDim.x + nxt));
+        // the next item is taken only once this item's loads are out and the
+        // softmax has begun this item (every role has released item k - 1): taken
+        // earlier, items would wait behind busy CTAs while others go idle
+        if (k >= 1 && !ptx::mbar_wait(item_free + (k - 1) % kRing, ((k - 1) / kRing) & 1, limit,
+                                      p.status))
+          limit = kWaitNsAfterFault;
+        publish(k + 1, (int)(gridDim.x + atomicAdd(p.sched, 1u)));
       }
       if (!kicked) ptx::mbar_arrive(kick);
     }
@@ -440,7 +471,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ================= TMA: each item's value tiles
     if (lane == 0) {
       int lv = 0;
-      if (!ptx::mbar_wait(kick, 0, limit, p.status)) limit = kWaitNsAfterFault;
       for (int k = 0;; ++k) {
         const volatile int* e = ring + (k % kRing) * kRingInts;
         const bool more = ring_wait(k, item_full, limit, p.status) && e[0] >= 0;
@@ -448,6 +478,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::mbar_arrive(item_free + k % kRing);
         if (!more) break;
         if (!g.work) continue;
+        // the first value tile waits until the first Q and key tile have landed
+        // (only here: the ring entries before it must still be released)
+        if (lv == 0 && !ptx::mbar_wait(kick, 0, limit, p.status)) limit = kWaitNsAfterFault;
         const int base_row = g.l * la.sum_T + g.t0;
         for (int j = 0; j < g.nq - g.qt; ++j) {
           const int s = lv % kStages;
