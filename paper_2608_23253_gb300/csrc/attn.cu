@@ -131,6 +131,33 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 
 __device__ __forceinline__ float neg_inf() { return __int_as_float(0xff800000); }
 
+// max of three (one instruction)
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Packed pairs of fp32 (one instruction per pair).
+__device__ __forceinline__ uint64_t f2_pack(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t r, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(r));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 
 // D (TMEM) (+)= A B with A read from TMEM (row i of A on lane i; for 16-bit
 // types two consecutive K elements per 32-bit column, the lower index in the
@@ -635,11 +662,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         // through shared memory; the buffer alternates with the tile)
         float mx[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) mx[i] = fmaxf(s[i], s[i + 8]);
-#pragma unroll
-        for (int i = 16; i < 64; ++i) mx[i & 7] = fmaxf(mx[i & 7], s[i]);
-        const float hmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                                 fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+        for (int i = 0; i < 8; ++i) {
+          mx[i] = max3f(s[i], s[i + 8], s[i + 16]);
+          mx[i] = max3f(mx[i], s[i + 24], s[i + 32]);
+          mx[i] = max3f(mx[i], s[i + 40], s[i + 48]);
+          mx[i] = fmaxf(mx[i], s[i + 56]);
+        }
+        const float hmax = max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[5]),
+                                 fmaxf(mx[6], mx[7]));
         xch[ch * kTile + r] = hmax;
         ptx::named_bar(pair_bar, 64);
         const float tmax = fmaxf(xch[r], xch[kTile + r]);
@@ -672,15 +702,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tc_fence_after();
         // P = 2^(s - m) in bf16 pairs: key 64 ch + 2 i + e -> P column 32 ch + i
         uint32_t pk[32];
-        float acc0 = 0.f, acc1 = 0.f;
+        const uint64_t sc2 = f2_pack(p.scale_log2, p.scale_log2), nm2 = f2_pack(-mnew, -mnew);
+        uint64_t acc2a = f2_pack(0.f, 0.f), acc2b = acc2a;
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          const float e0 = fast_ex2(fmaf(s[2 * i], p.scale_log2, -mnew));
-          const float e1 = fast_ex2(fmaf(s[2 * i + 1], p.scale_log2, -mnew));
-          acc0 += e0;
-          acc1 += e1;
+          float x0, x1;
+          f2_unpack(f2_fma(f2_pack(s[2 * i], s[2 * i + 1]), sc2, nm2), x0, x1);
+          const float e0 = fast_ex2(x0), e1 = fast_ex2(x1);
+          if (i & 1) {
+            acc2b = f2_add(acc2b, f2_pack(e0, e1));
+          } else {
+            acc2a = f2_add(acc2a, f2_pack(e0, e1));
+          }
           pk[i] = pack_bf16(e0, e1);
         }
+        float acc0, acc1, acc2, acc3;
+        f2_unpack(acc2a, acc0, acc1);
+        f2_unpack(acc2b, acc2, acc3);
+        acc0 += acc2;
+        acc1 += acc3;
         tmem_st32(tmem + lane_base + kColP + (uint32_t)pb * 64u + (uint32_t)(32 * ch), pk);
         ptx::tmem_wait_st();
         lsum = lsum * alpha + (acc0 + acc1);
