@@ -606,6 +606,10 @@ def measure_batched(name: str, dev, peaks: dict, steps: int) -> dict:
                             "frac_of_bf16_peak": flops / (mean_ms["score"] * 1e-3) / 1e12 / tf,
                             "ncu": tensor_pipe_record(name)},
            "steps": steps, "clocks": clocks.summary()}
+    if name == "cfg2":
+        # the layer's attention pass at batch 32 (the batch-1 one is in the main line)
+        out["attention_pass"] = attention_pass_entry(T, w, max(steps // 4, 5),
+                                                     out["decision_us"], peaks)
     del w, T
     torch.cuda.empty_cache()
     return out
@@ -653,10 +657,11 @@ def attention_pass_entry(T: Timing, w: Workload, n: int, decision_us: float, pea
             "separate_score_then_decision_us": decision_us,
             "attention_TFLOP/s": flops / (out["attention"] * 1e-6) / 1e12,
             "attention_frac_of_bf16_peak": flops / (out["attention"] * 1e-6) / 1e12 / tf,
-            "note": "e2s_attention over the pruning layer's 3 evidence layers (all 675 rows, "
-                    "causal, O and lse of every row); with_score adds the text rows' score a "
-                    "and its statistics in the same launch; attention_then_decision = "
-                    "e2s_decide_attn; separate = e2s_decide (its own score kernel)"}
+            "note": "e2s_attention over the pruning layer's evidence layers (every row of "
+                    "every image, causal, O and lse of every row); with_score adds the text "
+                    "rows' score a and its statistics in the same launch; "
+                    "attention_then_decision = e2s_decide_attn; separate = e2s_decide (its "
+                    "own score kernel)"}
 
 
 def run_ours(args, world, rank, local):
