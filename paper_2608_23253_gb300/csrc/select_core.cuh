@@ -18,11 +18,17 @@ namespace e2s {
 
 constexpr int kMaxCells = 64;
 
+constexpr int kSelDigitBits = 9;                  // radix digit of the threshold search
+constexpr int kSelBuckets = 1 << kSelDigitBits;
+constexpr int kSelCand = 32;                      // live keys one warp ranks directly
+
 struct SelectSmem {
   unsigned long long cell_best[kMaxCells];
-  uint32_t hist[3][256];   // one per radix pass, rotating (zeroed two passes ahead)
+  uint32_t hist[kSelBuckets];
+  uint32_t cand[kSelCand];
   uint32_t warp_tot[32];
   uint32_t w_and[32], w_or[32];   // per warp AND / OR of the keys
+  uint32_t sel[4];                // digit, its keys, keys still needed, candidates gathered
 };
 
 // Per-warp AND and OR of the keys a thread wrote (identity values for none);
@@ -105,12 +111,116 @@ __device__ __forceinline__ unsigned long long cell_key(float q, int n) {
   return ((unsigned long long)ordered_key(q) << 32) | (0xFFFFFFFFu - (uint32_t)n);
 }
 
+// Exact Kc-th largest of keys[0 .. NV) (0 < Kc < NV): its value thr and how
+// many of the keys equal to it are kept (need_eq).  Radix search from the
+// highest bit in which the keys differ (from the AND / OR that
+// publish_key_bits left in ss), kSelDigitBits bits per pass: a histogram of
+// the live keys' digit, one block-wide scan of it in descending order to find
+// the digit holding the remaining-th largest live key, and the live set
+// narrowed to that digit.  Once the digit's bucket holds at most kSelCand
+// keys, they are gathered and one warp ranks them against each other (each
+// lane compares its key with every gathered key, read as a shared-memory
+// broadcast), which gives the threshold directly; one or two 9-bit passes
+// usually leave that few.  Every thread of the block must call it.
+static __device__ void select_threshold(const uint32_t* keys, int NV, uint32_t Kc,
+                                        SelectSmem& ss, uint32_t& thr, uint32_t& need_eq) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nt = (int)blockDim.x, nw = nt >> 5;
+  uint32_t all_and = 0xFFFFFFFFu, all_or = 0u;
+  for (int w = 0; w < nw; ++w) {
+    all_and &= ss.w_and[w];
+    all_or |= ss.w_or[w];
+  }
+  const uint32_t diff = all_and ^ all_or;   // bits in which some keys differ
+  if (diff == 0u) {                         // every key is the same
+    thr = all_and;
+    need_eq = Kc;
+    return;
+  }
+  int top = 31 - __clz(diff);               // highest undecided bit
+  uint32_t mask = top == 31 ? 0u : (0xFFFFFFFFu << (top + 1));
+  uint32_t prefix = all_and & mask;         // live keys: (k & mask) == prefix
+  uint32_t remaining = Kc;
+  for (;;) {
+    const int shift = max(top - (kSelDigitBits - 1), 0);
+    const int nb = 1 << (top - shift + 1);
+    // the previous pass read the histogram and sel before its last barrier
+    for (int i = threadIdx.x; i < nb; i += nt) ss.hist[i] = 0u;
+    if (threadIdx.x == 0) ss.sel[3] = 0u;
+    __syncthreads();
+    for (int n = threadIdx.x; n < NV; n += nt) {
+      const uint32_t k = keys[n];
+      if ((k & mask) == prefix) atomicAdd(&ss.hist[(k >> shift) & (uint32_t)(nb - 1)], 1u);
+    }
+    __syncthreads();
+    // thread t owns the buckets of descending rank t*per .. t*per+per-1
+    const int per = (nb + nt - 1) / nt;
+    const int i0 = min((int)threadIdx.x * per, nb), i1 = min(i0 + per, nb);
+    uint32_t tot = 0;
+    for (int i = i0; i < i1; ++i) tot += ss.hist[nb - 1 - i];
+    uint32_t incl = tot;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (lane == 31) ss.warp_tot[warp] = incl;
+    __syncthreads();
+    uint32_t acc = incl - tot;
+    for (int w = 0; w < warp; ++w) acc += ss.warp_tot[w];
+    if (acc < remaining && remaining <= acc + tot) {   // exactly one thread
+      for (int i = i0; i < i1; ++i) {
+        const uint32_t h = ss.hist[nb - 1 - i];
+        if (acc + h >= remaining) {
+          ss.sel[0] = (uint32_t)(nb - 1 - i);
+          ss.sel[1] = h;
+          ss.sel[2] = remaining - acc;
+          break;
+        }
+        acc += h;
+      }
+    }
+    __syncthreads();
+    const uint32_t cnt = ss.sel[1];
+    prefix |= ss.sel[0] << shift;
+    mask |= (uint32_t)(nb - 1) << shift;
+    remaining = ss.sel[2];
+    if (shift == 0) {   // the live keys are all equal
+      thr = prefix;
+      need_eq = remaining;
+      return;
+    }
+    if (cnt <= (uint32_t)kSelCand) {
+      for (int n = threadIdx.x; n < NV; n += nt) {
+        const uint32_t k = keys[n];
+        if ((k & mask) == prefix) ss.cand[atomicAdd(&ss.sel[3], 1u)] = k;
+      }
+      __syncthreads();
+      if (warp == 0) {
+        const uint32_t mine = (uint32_t)lane < cnt ? ss.cand[lane] : 0u;
+        uint32_t gt = 0, eq = 0;
+        for (uint32_t j = 0; j < cnt; ++j) {   // every lane reads the same word
+          const uint32_t o = ss.cand[j];
+          gt += o > mine ? 1u : 0u;
+          eq += o == mine ? 1u : 0u;
+        }
+        // the remaining-th largest live key (equal keys write the same values)
+        if ((uint32_t)lane < cnt && gt < remaining && remaining <= gt + eq) {
+          ss.sel[0] = mine;
+          ss.sel[1] = remaining - gt;
+        }
+      }
+      __syncthreads();
+      thr = ss.sel[0];
+      need_eq = ss.sel[1];
+      return;
+    }
+    top = shift - 1;
+  }
+}
+
 // Steps 3-4 over the ordered keys of q~ (keys[0 .. NV) in shared memory).
-// 3. exact K-th largest key by a 4-pass, 8-bit radix select: one histogram
-//    per pass (three buffers in rotation, so a pass needs a single barrier),
-//    and every warp scans the histogram itself to find the digit; a pass
-//    whose 8 bits are the same in every key (from the AND / OR of all keys
-//    that publish_key_bits left in ss) is skipped;
+// 3. exact K-th largest key (select_threshold);
 // 4. ascending emission: each thread owns a contiguous run of slots; one
 //    block-wide exclusive scan of (count above the threshold, count equal to
 //    it), packed in 16-bit halves, gives every kept slot its position.  Among
@@ -123,64 +233,7 @@ static __device__ void select_rank_emit(const uint32_t* keys, int NV, int K, Sel
   const bool keep_all = Kc == NV;
   uint32_t thr = 0, need_eq = 0;
   if (!keep_all && Kc > 0) {
-    uint32_t all_and = 0xFFFFFFFFu, all_or = 0u;
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
-      all_and &= ss.w_and[w];
-      all_or |= ss.w_or[w];
-    }
-    const uint32_t same = ~(all_and ^ all_or);   // bits equal in every key
-    for (int i = threadIdx.x; i < 2 * 256; i += blockDim.x) (&ss.hist[0][0])[i] = 0u;
-    __syncthreads();
-    uint32_t prefix = 0, mask = 0, remaining = (uint32_t)Kc;
-    int ex = 0;   // executed passes: executed pass e uses buffer e % 3
-    for (int pass = 0; pass < 4; ++pass) {
-      const int shift = 24 - 8 * pass;
-      if (((same >> shift) & 255u) == 255u) {   // every key has this digit
-        prefix |= all_and & (255u << shift);
-        mask |= 255u << shift;
-        continue;
-      }
-      uint32_t* hist = ss.hist[ex % 3];
-      for (int n = threadIdx.x; n < NV; n += blockDim.x) {
-        const uint32_t k = keys[n];
-        if ((k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1u);
-      }
-      __syncthreads();
-      // the buffer of two executed passes ahead was last read before this barrier
-      for (int i = threadIdx.x; i < 256; i += blockDim.x) ss.hist[(ex + 2) % 3][i] = 0u;
-      ++ex;
-      // digit holding the remaining-th largest key, buckets from 255 down
-      uint32_t c[8], tot = 0;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        c[i] = hist[255 - 8 * lane - i];
-        tot += c[i];
-      }
-      uint32_t incl = tot;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
-      }
-      uint32_t excl = incl - tot, digit = 0, rem = 0;
-      const bool here = excl < remaining && remaining <= incl;
-      if (here) {
-        for (int i = 0; i < 8; ++i) {
-          if (excl + c[i] >= remaining) {
-            digit = (uint32_t)(255 - 8 * lane - i);
-            rem = remaining - excl;
-            break;
-          }
-          excl += c[i];
-        }
-      }
-      const int src = __ffs(__ballot_sync(0xffffffffu, here)) - 1;
-      prefix |= __shfl_sync(0xffffffffu, digit, src) << shift;
-      remaining = __shfl_sync(0xffffffffu, rem, src);
-      mask |= 255u << shift;
-    }
-    thr = prefix;
-    need_eq = remaining;
+    select_threshold(keys, NV, (uint32_t)Kc, ss, thr, need_eq);
   }
 
   // 4. emit ascending indices
