@@ -1,7 +1,8 @@
 // Compaction of the retained rows: system rows, the kept visual rows and the
 // text rows of every image are gathered, in order, into the shortened
 // sequence that the next decoder layer consumes.  One warp per (tensor,
-// output row); 16-byte streaming loads and stores, fully coalesced.
+// output row); 16-byte streaming loads and stores, fully coalesced; each
+// CTA first stages every image's constants in shared memory.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -13,7 +14,6 @@ namespace e2s {
 namespace {
 
 constexpr int kCompactThreads = 256;
-constexpr int kRowVec = 16;   // 16-byte vectors per lane in flight
 constexpr long long kPrefetchBytes = 48ll << 20;   // candidate rows prefetched into L2
 
 struct TensorSet {
@@ -33,14 +33,44 @@ __device__ __forceinline__ int out_image(const LayoutArgs& la, const int32_t* ke
   return lo;
 }
 
+// Per-image constants of the gather: the image's first output row, its
+// system / visual / text counts, its keep list and its first input row.
+struct ImgRows {
+  int out0, S, NV, NT, ko, Kb, tok;
+};
+constexpr int kTabImages = 256;   // images whose constants a CTA stages in shared memory
+
+__device__ __forceinline__ ImgRows img_rows(const LayoutArgs& la, const int32_t* keep_off, int b) {
+  ImgRows t;
+  t.S = __ldg(la.n_sys + b);
+  t.NV = __ldg(la.n_vis + b);
+  t.NT = __ldg(la.n_text + b);
+  t.ko = __ldg(keep_off + b);
+  t.Kb = __ldg(keep_off + b + 1) - t.ko;
+  t.tok = __ldg(la.tok_off + b);
+  t.out0 = t.tok - __ldg(la.vis_off + b) + t.ko;
+  return t;
+}
+
+// Every image's constants into shared memory (whole block; la.B <= kTabImages).
+__device__ __forceinline__ void stage_images(const LayoutArgs& la, const int32_t* keep_off,
+                                             ImgRows* tab) {
+  for (int b = threadIdx.x; b < la.B; b += blockDim.x) tab[b] = img_rows(la, keep_off, b);
+  __syncthreads();
+}
+
 // One (tensor, output row) pair per warp, grid-stride.  visual < 0: every
 // row; visual == 0: system and text rows only; visual == 1: kept visual rows
-// only.
+// only.  tab (nullable): the images' constants in shared memory, so that a
+// pair's source row costs a shared-memory search instead of a chain of
+// dependent global loads.
+// RV: 16-byte vectors per lane in flight (RV * 512 bytes of a row per warp).
+template <int RV>
 __device__ __forceinline__ void compact_rows(const LayoutArgs& la, const int32_t* keep_idx,
                                              const int32_t* keep_off, int n_tensors,
                                              const TensorSet& ts, int32_t* pos_ids,
                                              long long total_rows, uint32_t* status, int visual,
-                                             bool spread) {
+                                             bool spread, const ImgRows* tab) {
   const int lane = threadIdx.x & 31;
   const long long warps = (long long)gridDim.x * (blockDim.x >> 5);
   // with no tensors the pass still writes the position ids
@@ -51,14 +81,22 @@ __device__ __forceinline__ void compact_rows(const LayoutArgs& la, const int32_t
   // neighbouring rows stay in one CTA (DRAM locality)
   const long long first = spread ? (long long)(threadIdx.x >> 5) * gridDim.x + blockIdx.x
                                  : ((long long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const bool narrow = pairs < (1ll << 31);   // 32-bit pair arithmetic
   for (long long pr = first; pr < pairs; pr += warps) {
-    const int tix = (int)(pr / total_rows);
+    const int tix = narrow ? (int)((uint32_t)pr / (uint32_t)total_rows) : (int)(pr / total_rows);
     const int r = (int)(pr - (long long)tix * total_rows);
-    const int b = out_image(la, keep_off, r);
-    const int S = __ldg(la.n_sys + b), NV = __ldg(la.n_vis + b), NT = __ldg(la.n_text + b);
-    const int ko = __ldg(keep_off + b);
-    const int Kb = __ldg(keep_off + b + 1) - ko;
-    const int out0 = __ldg(la.tok_off + b) - __ldg(la.vis_off + b) + ko;
+    ImgRows t;
+    if (tab != nullptr) {   // largest b with tab[b].out0 <= r
+      int lo = 0, hi = la.B - 1;
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (tab[mid].out0 <= r) lo = mid; else hi = mid - 1;
+      }
+      t = tab[lo];
+    } else {
+      t = img_rows(la, keep_off, out_image(la, keep_off, r));
+    }
+    const int S = t.S, NV = t.NV, NT = t.NT, ko = t.ko, Kb = t.Kb, out0 = t.out0;
     const int u = r - out0;
     const bool is_vis = u >= S && u < S + Kb;
     if (visual >= 0 && is_vis != (visual == 1)) continue;
@@ -79,21 +117,21 @@ __device__ __forceinline__ void compact_rows(const LayoutArgs& la, const int32_t
     }
     if (tix == 0 && lane == 0 && pos_ids) pos_ids[r] = src_local;
     if (n_tensors == 0) continue;
-    const long long src_row = (long long)__ldg(la.tok_off + b) + src_local;
+    const long long src_row = (long long)t.tok + src_local;
     const int64_t rb = ts.row_bytes[tix];
     const uint4* s4 = reinterpret_cast<const uint4*>(ts.src[tix] + src_row * rb);
     uint4* d4 = reinterpret_cast<uint4*>(ts.dst[tix] + (long long)r * rb);
     const int n16 = (int)(rb >> 4);
     // up to 8 KiB of the row in flight per warp: all loads first, then stores
-    for (int base = 0; base < n16; base += 32 * kRowVec) {
-      uint4 x[kRowVec];
+    for (int base = 0; base < n16; base += 32 * RV) {
+      uint4 x[RV];
 #pragma unroll
-      for (int v = 0; v < kRowVec; ++v) {
+      for (int v = 0; v < RV; ++v) {
         const int i = base + v * 32 + lane;
         if (i < n16) x[v] = __ldcs(s4 + i);
       }
 #pragma unroll
-      for (int v = 0; v < kRowVec; ++v) {
+      for (int v = 0; v < RV; ++v) {
         const int i = base + v * 32 + lane;
         if (i < n16) __stcs(d4 + i, x[v]);
       }
@@ -123,21 +161,28 @@ __device__ __forceinline__ void prefetch_visual_rows(const LayoutArgs& la, int n
 // keep_idx; the caller guarantees that the sources and keep_off were complete
 // before that kernel's predecessor started.  prefetch != 0 (with early): the
 // candidate visual rows are also prefetched into L2 while waiting.
+template <int RV>
 __global__ void __launch_bounds__(kCompactThreads)
     compact_kernel(const LayoutArgs la, const int32_t* __restrict__ keep_idx,
                    const int32_t* __restrict__ keep_off, int n_tensors, const TensorSet ts,
                    int32_t* __restrict__ pos_ids, long long total_rows, uint32_t* status,
                    int early, int prefetch) {
+  __shared__ ImgRows tab_s[kTabImages];
+  const ImgRows* tab = la.B <= kTabImages ? tab_s : nullptr;
   pdl_launch_dependents();
   if (early) {
     if (prefetch) prefetch_visual_rows(la, n_tensors, ts);
-    compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, 0, false);
+    if (tab) stage_images(la, keep_off, tab_s);
+    compact_rows<RV>(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, 0, false,
+                 tab);
     pdl_wait();   // keep_idx comes from the previous kernel
-    compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, 1,
-                 prefetch != 0);
+    compact_rows<RV>(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, 1,
+                 prefetch != 0, tab);
   } else {
     pdl_wait();
-    compact_rows(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, -1, false);
+    if (tab) stage_images(la, keep_off, tab_s);
+    compact_rows<RV>(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, -1, false,
+                 tab);
   }
 }
 
@@ -169,9 +214,18 @@ cudaError_t launch_compact(const LayoutArgs& la, const int32_t* keep_idx, const 
   const int warps_per_block = kCompactThreads / 32;
   long long blocks = (pairs + warps_per_block - 1) / warps_per_block;
   blocks = std::min<long long>(blocks, (long long)sm_count() * 16);
-  return launch_kernel(compact_kernel, dim3((unsigned)std::max<long long>(blocks, 1)),
-                       dim3(kCompactThreads), 0, st, 0, true, la, keep_idx, keep_off, n_tensors, ts,
-                       pos_ids, total_rows, status, early, prefetch);
+  const dim3 grid((unsigned)std::max<long long>(blocks, 1));
+  // 8 KiB of a row per warp (112 registers, two CTAs per SM) when there are
+  // only a few rows per warp slot and nothing overlaps the copy; otherwise
+  // 4 KiB per warp (66 registers, three CTAs per SM), which measured faster
+  // in the whole step and on large batches
+  if (!early && pairs <= (long long)sm_count() * 64)
+    return launch_kernel(compact_kernel<16>, grid, dim3(kCompactThreads), 0, st, 0, true, la,
+                         keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, early,
+                         prefetch);
+  return launch_kernel(compact_kernel<8>, grid, dim3(kCompactThreads), 0, st, 0, true, la,
+                       keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, early,
+                       prefetch);
 }
 
 }  // namespace e2s
