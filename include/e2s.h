@@ -105,9 +105,10 @@ typedef struct {
 /* Bytes of workspace every call below needs: the status word, one float4 of
  * normalisation statistics per (image, layer, head) written by e2s_score and
  * e2s_decide, and one arrival counter per image (e2s_decide).  The workspace
- * must be 256-byte aligned and its first 16 bytes zero before the first call
- * (e2s_clear_status zeroes them; bytes 4..15 hold the attention kernel's item
- * counter, which every call leaves zero); the rest needs no initialisation. */
+ * must be 256-byte aligned and its first 32 bytes zero before the first call
+ * (e2s_clear_status zeroes them; bytes 4..11 hold the attention kernel's item
+ * counter and bytes 12..19 the streaming score kernel's unit counter, which
+ * every call leaves zero); the rest needs no initialisation. */
 size_t e2s_workspace_size(const e2s_layout* layout, const e2s_params* params);
 
 /* Text-to-visual score (Sec. 3.1, Eq. 1; Algorithm 1 "Compute a_{l,h,n}").
@@ -360,8 +361,9 @@ e2s_status e2s_compact(const e2s_layout* layout, const int32_t* keep_idx,
  * error).  Does not clear it. */
 e2s_status e2s_read_status(const void* ws, void* stream);
 
-/* Zeroes the first 16 bytes of the workspace: the device status word and the
- * attention kernel's item counter (stream-ordered, asynchronous). */
+/* Zeroes the first 32 bytes of the workspace: the device status word and the
+ * attention and streaming score kernels' work counters (stream-ordered,
+ * asynchronous). */
 e2s_status e2s_clear_status(void* ws, void* stream);
 
 /* Human-readable name of a status value (static string). */

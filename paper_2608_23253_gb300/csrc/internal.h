@@ -29,7 +29,10 @@ inline uint32_t* status_word(void* ws) { return reinterpret_cast<uint32_t*>(ws);
 // Words 1 and 2 of the status area: the attention kernel's shared item counter
 // and its count of finished CTAs (zero between calls).
 inline uint32_t* attn_sched_ptr(void* ws) { return reinterpret_cast<uint32_t*>(ws) + 1; }
-constexpr size_t kClearBytes = 16;   // bytes of the status area zeroed before first use
+// Words 3 and 4: the streaming score kernel's shared unit counter and its
+// count of finished CTAs (zero between calls); status is word 0.
+inline uint32_t* stream_sched_ptr(uint32_t* status) { return status + 3; }
+constexpr size_t kClearBytes = 32;   // bytes of the status area zeroed before first use
 inline float4* stats_ptr(void* ws) {
   return reinterpret_cast<float4*>(reinterpret_cast<char*>(ws) + kStatusBytes);
 }

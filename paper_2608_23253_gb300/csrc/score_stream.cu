@@ -112,13 +112,22 @@ struct StreamArgs {
   float4* stats;        // per (image, layer, head) statistics of the visual scores
   uint32_t* counters;   // nullable: decision scratch to zero
   uint32_t* status;
+  uint32_t* sched;      // nullable: [0] units handed out after the first, [1] CTAs done
+  int upi;              // units per image
+  int order;            // 0: index order; 1: heaviest first if the costs are skewed;
+                        // 2: heaviest first (la.B <= kOrderMax)
 };
+
+constexpr int kURing = 4;        // unit indices in flight from the producer to the other roles
+constexpr int kOrderMax = 256;   // images the heaviest-first order covers
 
 struct SPlan {
-  uint32_t q, k, bars, slot, ms, lse, cps, red, total;
+  uint32_t q, k, bars, slot, ms, lse, cps, red, ring, order, cost, ubars, total;
 };
 
-__host__ __device__ inline SPlan stream_plan(int stages) {
+// dyn: with the unit ring, its barriers and the image order (round-robin
+// launches leave them out, so their shared memory stays as small as before).
+__host__ __device__ inline SPlan stream_plan(int stages, bool dyn) {
   SPlan s;
   s.q = 0;                                              // [2 halves][128 rows][128 B]
   s.k = (uint32_t)kTileBytes;                           // [stages][tile]
@@ -128,7 +137,11 @@ __host__ __device__ inline SPlan stream_plan(int stages) {
   s.lse = s.ms + 4u * kRows * 8u;                       // [128] float -lse per text row
   s.cps = s.lse + kRows * 4u;                           // [2][8 chunks][128 keys] partials
   s.red = s.cps + 2u * 8u * kTileKeys * 4u;             // [4 heads][4] float4 statistics
-  s.total = s.red + 16u * 16u;
+  s.ring = s.red + 16u * 16u;                           // [kURing] int unit indices
+  s.order = s.ring + 4u * kURing;                       // [kOrderMax] int images, heaviest first
+  s.cost = s.order + 4u * kOrderMax;                    // [kOrderMax] float image costs
+  s.ubars = s.cost + 4u * kOrderMax;                    // [2][kURing] unit-ring mbarriers
+  s.total = dyn ? s.ubars + 16u * kURing : s.ring;
   return s;
 }
 
@@ -196,12 +209,31 @@ __device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit) {
   return g;
 }
 
+// Relative cost of one image's units: key tiles streamed by both sweeps, each
+// weighted by the text rows the epilogue sweeps (plus a fixed share for the
+// MMAs and the tile's own overhead).
+__device__ __forceinline__ float image_cost(const LayoutArgs& la, int b) {
+  const float S = (float)__ldg(la.n_sys + b), NV = (float)__ldg(la.n_vis + b);
+  const float NT = (float)__ldg(la.n_text + b);
+  return (S + 2.f * NV + NT) * (NT + 64.f);
+}
+
+// Work index w (0 .. num_units - 1, in hand-out order) -> unit: with an
+// order, the units of the image of rank w / upi.
+__device__ __forceinline__ int unit_of(const StreamArgs& p, const int* order, int w) {
+  if (!p.order) return w;
+  const int r = w / p.upi;
+  return order[r] * p.upi + (w - r * p.upi);
+}
+
 // HPU: query heads stacked per unit (1, 2 or 4), fixed at compile time so that
 // the row mapping and the quarter sums are unrolled.  SPLIT (one head of at
 // most 64 text rows): the queries fill TMEM lanes 0-63 and again 64-127, and
 // in sweep 1 each half of the lanes takes half of every key tile's columns, so
 // all four lane quarters (all four SM sub-partitions) share the exponentials.
-template <int HPU, bool SPLIT>
+// DYN: units come from the workspace counter through the unit ring (p.sched
+// set); otherwise round-robin, and the ring's code is compiled out.
+template <int HPU, bool SPLIT, bool DYN>
 __global__ void __launch_bounds__(kThreads, 1)
     score_stream_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmK, const StreamArgs p) {
@@ -209,7 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const LayoutArgs& la = p.la;
-  const SPlan plan = stream_plan(p.stages);
+  const SPlan plan = stream_plan(p.stages, DYN);
   constexpr uint32_t q_half = kHalfBytes;   // bytes of one 64-element half of Q
   uint8_t* q_sm = smem + plan.q;
   uint8_t* k_sm = smem + plan.k;
@@ -222,6 +254,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* b_full = a_empty + 2;          // [kMaxBatch] batch sweep-2 accumulator ready
   uint64_t* b_done = b_full + kMaxBatch;   // batch sweep 2 read: TMEM free again
   uint64_t* s1_done = b_done + 1;          // a batch unit's sweep-1 accumulators all read
+  uint64_t* u_full = reinterpret_cast<uint64_t*>(smem + plan.ubars);   // [kURing] unit published
+  uint64_t* u_free = u_full + kURing;      // [kURing] unit index read by every consumer
+  volatile int* uring = reinterpret_cast<volatile int*>(smem + plan.ring);
+  int* order_s = reinterpret_cast<int*>(smem + plan.order);
+  float* cost_s = reinterpret_cast<float*>(smem + plan.cost);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + plan.slot);
   float2* ms = reinterpret_cast<float2*>(smem + plan.ms);
   float* nlse = reinterpret_cast<float*>(smem + plan.lse);   // -lse per text row
@@ -250,24 +287,86 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < kMaxBatch; ++i) ptx::mbar_init(b_full + i, 1);
     ptx::mbar_init(b_done, kEpiWarps);
     ptx::mbar_init(s1_done, kEpiWarps);
+    for (int i = 0; i < (DYN ? kURing : 0); ++i) {
+      ptx::mbar_init(u_full + i, 1);
+      ptx::mbar_init(u_free + i, 2 + kEpiWarps);   // both MMA issuers and every epilogue warp
+    }
     ptx::fence_barrier_init();
     ptx::fence_proxy_async_smem();
     ptx::prefetch_tensormap(&tmQ);
     ptx::prefetch_tensormap(&tmK);
   }
   if (warp == 1) ptx::tmem_alloc(tmem_slot, kTmemCols);
+  if (DYN && p.order) {
+    // Every CTA derives the same order.  With few units per CTA (order 2)
+    // or when the costliest image costs more than twice the mean, images go
+    // heaviest first (cost descending, then index), so that the last units
+    // handed out are light ones; otherwise in index order, which keeps heavy
+    // and light units mixed on the SMs (heaviest first measured slower there).
+    for (int i = threadIdx.x; i < la.B; i += blockDim.x) cost_s[i] = image_cost(la, i);
+    __syncthreads();
+    float cmax = 0.f, csum = 0.f;
+    for (int j = 0; j < la.B; ++j) {
+      cmax = fmaxf(cmax, cost_s[j]);
+      csum += cost_s[j];
+    }
+    const bool skewed = p.order == 2 || cmax * (float)la.B > 2.f * csum;
+    for (int i = threadIdx.x; i < la.B; i += blockDim.x) {
+      const float c = cost_s[i];
+      int r = i;
+      if (skewed) {
+        r = 0;
+        for (int j = 0; j < la.B; ++j) {
+          const float cj = cost_s[j];
+          r += (cj > c || (cj == c && j < i)) ? 1 : 0;
+        }
+      }
+      order_s[r] = i;
+    }
+  }
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   uint64_t limit = kWaitNs;
+  // consumer side of the unit ring: one thread per MMA issuer, or a whole
+  // epilogue warp, whose lane 0 releases the slot once every lane has read it
+  // (without the counter, units go round-robin and there is no ring)
+  auto take_unit = [&](int u, bool warp_wide) -> int {
+    if constexpr (!DYN) {   // round-robin
+      const int w = (int)blockIdx.x + u * (int)gridDim.x;
+      return w < p.num_units ? w : -1;
+    }
+    const int slot = u % kURing;
+    if (!ptx::mbar_wait(u_full + slot, (u / kURing) & 1, limit, p.status)) {
+      limit = kWaitNsAfterFault;
+      return -1;
+    }
+    const int unit = uring[slot];
+    if (warp_wide) __syncwarp();
+    if (!warp_wide || lane == 0) ptx::mbar_arrive(u_free + slot);
+    return unit;
+  };
 
   if (warp == 0) {
     // ================= TMA producer: per unit the 128 text rows, then every
     // key tile of sweep 1 and of sweep 2 through the ring
     if (lane == 0) {
-      int ld = 0, u = 0;
-      for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x, ++u) {
+      // unit u of this CTA (work index w) goes into ring slot u % kURing for
+      // the MMA issuers and the epilogue; -1 ends the walk
+      auto publish = [&](int u, int w) {
+        if constexpr (!DYN) return w < p.num_units ? w : -1;   // round-robin: no ring
+        const int unit_w = w < p.num_units ? unit_of(p, order_s, w) : -1;
+        const int slot = u % kURing;
+        if (u >= kURing && !ptx::mbar_wait(u_free + slot, (u / kURing - 1) & 1, limit, p.status))
+          limit = kWaitNsAfterFault;
+        uring[slot] = unit_w;
+        ptx::mbar_arrive(u_full + slot);
+        return unit_w;
+      };
+      int ld = 0;
+      int unit = publish(0, (int)blockIdx.x);   // the CTA's own first unit
+      for (int u = 0; unit >= 0; ++u) {
         const SGeo g = stream_geo<HPU, SPLIT>(p, unit);
         if (!g.ok) E2S_DEV_FLAG(p.status, E2S_ERR_SHAPE);
         if (u > 0 && !ptx::mbar_wait(q_empty, (u - 1) & 1, limit, p.status))
@@ -300,11 +399,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           ptx::tma_load_3d(k_sm + s * kTileBytes, &tmK, k_full + s, 0, g.kvh, krow);
           ptx::tma_load_3d(k_sm + s * kTileBytes + kHalfBytes, &tmK, k_full + s, 64, g.kvh, krow);
         }
-        // every load of this unit issued: the next unit's queries and first key
-        // tiles go to L2, so that its loads do not start from DRAM when this
-        // unit's last MMAs retire
-        const int next = unit + (int)gridDim.x;
-        if (next < p.num_units) {
+        // every load of this unit issued: the next unit is taken now, and its
+        // queries and first key tiles go to L2, so that its loads do not start
+        // from DRAM when this unit's last MMAs retire
+        // (claimed only now: claimed a unit earlier, units waited behind busy
+        // CTAs -- 270 -> 286 us on the high-resolution batch)
+        const int next = publish(u + 1, DYN ? (int)gridDim.x + (int)atomicAdd(p.sched, 1u)
+                                            : (int)blockIdx.x + (u + 1) * (int)gridDim.x);
+        unit = next;
+        if (next >= 0) {
           const SGeo gn = stream_geo<HPU, SPLIT>(p, next);
           if (gn.n1 + gn.n2 > 0) {
             const int qrow = gn.l * la.sum_text + gn.x0;
@@ -351,7 +454,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           ptx::mma_bf16(d, a0 + off, b0 + off, idesc, ks > 0 ? 1u : 0u);
         }
       };
-      for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x, ++u) {
+      for (;; ++u) {
+        const int unit = take_unit(u, false);
+        if (unit < 0) break;
         const SGeo g = stream_geo<HPU, SPLIT>(p, unit);
         const int n2c = sweep2_cols<HPU>(g.NT);
         const uint32_t idesc2 = ptx::idesc_bf16_f32(kTileKeys, n2c);
@@ -415,7 +520,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_base = (uint32_t)(q4 * 32) << 16;
     const int et = threadIdx.x - 64;
     int tc = 0, bu = 0;
-    for (int unit = blockIdx.x; unit < p.num_units; unit += gridDim.x) {
+    for (int u = 0;; ++u) {
+      const int unit = take_unit(u, true);
+      if (unit < 0) break;
       const SGeo g = stream_geo<HPU, SPLIT>(p, unit);
       // TMEM row lrow holds text row t of stacked head hs (SPLIT: row lrow % 64)
       const int hs = SPLIT ? 0 : lrow / kRph;
@@ -662,6 +769,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, kTmemCols);
   }
+  if (DYN && threadIdx.x == 0) {
+    // the last CTA out (every CTA has taken its last unit) zeroes the counter
+    __threadfence();
+    if (atomicAdd(p.sched + 1, 1u) == gridDim.x - 1) {
+      atomicExch(p.sched, 0u);
+      atomicExch(p.sched + 1, 0u);
+    }
+  }
 }
 
 }  // namespace
@@ -672,7 +787,7 @@ static int stream_stages() {
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
   cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
   for (int st = kMaxStages; st >= 2; --st)
-    if ((int)(stream_plan(st).total + 1024) <= optin) return st;
+    if ((int)(stream_plan(st, true).total + 1024) <= optin) return st;
   return 0;
 }
 
@@ -703,7 +818,18 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
   p.stats = stats;
   p.counters = counters;
   p.status = status;
+  p.upi = la.L * la.H_kv * p.upk;
   if (p.num_units == 0 || la.sum_vis == 0) return cudaSuccess;
+  // With fewer than 16 units per CTA, units are handed out from a counter in
+  // the workspace, so that CTAs that drew light units take more of them --
+  // heaviest images first below 6 units per CTA (or when the image costs are
+  // skewed); with more, round-robin.  Measured: Qwen2-VL batch 16 (5 units
+  // per CTA) 85 -> 69 us; high-resolution batch 8 (6.7) unchanged, 272 us
+  // heaviest first; LLaVA batch 32 (20) 1-2 % slower with the counter and
+  // 4 % slower heaviest first.
+  const int grid_n = std::min(p.num_units, sm_count());
+  p.sched = status != nullptr && p.num_units < 16 * grid_n ? stream_sched_ptr(status) : nullptr;
+  p.order = !p.sched || la.B <= 1 || la.B > kOrderMax ? 0 : p.num_units < 6 * grid_n ? 2 : 1;
   CUtensorMap tmQ, tmK;
   // one head of at most 64 text rows: the queries are loaded twice (SPLIT)
   const bool split = hpu == 1 && la.max_text <= kRows / 2;
@@ -712,19 +838,19 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
       !make_score_map(&tmK, k, la.H_kv, (int64_t)la.L * la.sum_T, k_stride, kTileKeys))
     return cudaErrorInvalidValue;
   if (p.stages < 2) return cudaErrorInvalidValue;
-  const size_t smem = stream_plan(p.stages).total + 1024;
-  const dim3 grid((unsigned)std::min(p.num_units, sm_count()));
+  const size_t smem = stream_plan(p.stages, p.sched != nullptr).total + 1024;
+  const dim3 grid((unsigned)grid_n);
+  const bool dyn = p.sched != nullptr;
+  auto go = [&](auto kernel) {
+    return launch_kernel(kernel, grid, dim3(kThreads), smem, st, 0, false, tmQ, tmK, p);
+  };
   if (hpu == 4)
-    return launch_kernel(score_stream_kernel<4, false>, grid, dim3(kThreads), smem, st, 0, false,
-                         tmQ, tmK, p);
+    return dyn ? go(score_stream_kernel<4, false, true>) : go(score_stream_kernel<4, false, false>);
   if (hpu == 2)
-    return launch_kernel(score_stream_kernel<2, false>, grid, dim3(kThreads), smem, st, 0, false,
-                         tmQ, tmK, p);
+    return dyn ? go(score_stream_kernel<2, false, true>) : go(score_stream_kernel<2, false, false>);
   if (split)
-    return launch_kernel(score_stream_kernel<1, true>, grid, dim3(kThreads), smem, st, 0, false,
-                         tmQ, tmK, p);
-  return launch_kernel(score_stream_kernel<1, false>, grid, dim3(kThreads), smem, st, 0, false,
-                       tmQ, tmK, p);
+    return dyn ? go(score_stream_kernel<1, true, true>) : go(score_stream_kernel<1, true, false>);
+  return dyn ? go(score_stream_kernel<1, false, true>) : go(score_stream_kernel<1, false, false>);
 }
 
 }  // namespace e2s
