@@ -52,6 +52,7 @@ constexpr int kHalfBytes = 128 * 128;         // 128 rows x 64 bf16
 constexpr int kTileBytes = 2 * kHalfBytes;    // one 128 x 128 bf16 operand
 constexpr int kMaxStages = 8;                 // K ring depth: as many as shared memory holds
 constexpr int kMaxBatch = 8;                  // sweep-2 tiles of a batch unit (whole TMEM)
+constexpr int kQBufs = 2;                     // query buffers at most (p.qbufs: 1 or 2)
 constexpr int kTmemCols = 512;                // two 128-column accumulators, or a batch
 constexpr int kEpiWarps = 16;
 constexpr int kEpiThreads = 32 * kEpiWarps;
@@ -114,6 +115,7 @@ struct StreamArgs {
   uint32_t* status;
   uint32_t* sched;      // nullable: [0] units handed out after the first, [1] CTAs done
   int upi;              // units per image
+  int qbufs;            // query buffers: 2 lets the next unit's queries land early
   int order;            // 0: index order; 1: heaviest first if the costs are skewed;
                         // 2: heaviest first (la.B <= kOrderMax)
 };
@@ -127,12 +129,12 @@ struct SPlan {
 
 // dyn: with the unit ring, its barriers and the image order (round-robin
 // launches leave them out, so their shared memory stays as small as before).
-__host__ __device__ inline SPlan stream_plan(int stages, bool dyn) {
+__host__ __device__ inline SPlan stream_plan(int stages, bool dyn, int qbufs) {
   SPlan s;
-  s.q = 0;                                              // [2 halves][128 rows][128 B]
-  s.k = (uint32_t)kTileBytes;                           // [stages][tile]
+  s.q = 0;                                              // [kQBufs][2 halves][128 rows][128 B]
+  s.k = (uint32_t)(qbufs * kTileBytes);                 // [stages][tile]
   s.bars = s.k + (uint32_t)stages * kTileBytes;         // mbarriers, see the kernel
-  s.slot = s.bars + 8u * (uint32_t)(2 + 2 * kMaxStages + 4 + kMaxBatch + 2);
+  s.slot = s.bars + 8u * (uint32_t)(2 * kQBufs + 2 * kMaxStages + 4 + kMaxBatch + 2);
   s.ms = (s.slot + 16u + 15u) & ~15u;                   // [4][128] float2 (max, sum)
   s.lse = s.ms + 4u * kRows * 8u;                       // [128] float -lse per text row
   s.cps = s.lse + kRows * 4u;                           // [2][8 chunks][128 keys] partials
@@ -241,13 +243,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const LayoutArgs& la = p.la;
-  const SPlan plan = stream_plan(p.stages, DYN);
+  const SPlan plan = stream_plan(p.stages, DYN, p.qbufs);
   constexpr uint32_t q_half = kHalfBytes;   // bytes of one 64-element half of Q
   uint8_t* q_sm = smem + plan.q;
   uint8_t* k_sm = smem + plan.k;
-  uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + plan.bars);
-  uint64_t* q_empty = q_full + 1;
-  uint64_t* k_full = q_empty + 1;          // [kMaxStages]
+  uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + plan.bars);   // [kQBufs]
+  uint64_t* q_empty = q_full + kQBufs;     // [kQBufs]
+  uint64_t* k_full = q_empty + kQBufs;     // [kMaxStages]
   uint64_t* k_empty = k_full + kMaxStages; // [kMaxStages]
   uint64_t* a_full = k_empty + kMaxStages; // [2] accumulator buffer ready
   uint64_t* a_empty = a_full + 2;          // [2] accumulator buffer read
@@ -274,8 +276,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       p.counters[i] = 0u;
 
   if (warp == 0 && lane == 0) {
-    ptx::mbar_init(q_full, 1);
-    ptx::mbar_init(q_empty, 2);   // one commit per MMA issuer
+    for (int i = 0; i < kQBufs; ++i) {
+      ptx::mbar_init(q_full + i, 1);
+      ptx::mbar_init(q_empty + i, 2);   // one commit per MMA issuer
+    }
     for (int i = 0; i < kMaxStages; ++i) {
       ptx::mbar_init(k_full + i, 1);
       ptx::mbar_init(k_empty + i, 1);
@@ -369,22 +373,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int u = 0; unit >= 0; ++u) {
         const SGeo g = stream_geo<HPU, SPLIT>(p, unit);
         if (!g.ok) E2S_DEV_FLAG(p.status, E2S_ERR_SHAPE);
-        if (u > 0 && !ptx::mbar_wait(q_empty, (u - 1) & 1, limit, p.status))
+        // unit u's queries go into buffer u % qbufs once the unit qbufs back is
+        // done with it (with two, they land while the previous unit finishes)
+        const int qb = u % p.qbufs;
+        uint8_t* q_dst = q_sm + qb * kTileBytes;
+        if (u >= p.qbufs && !ptx::mbar_wait(q_empty + qb, (u / p.qbufs - 1) & 1, limit, p.status))
           limit = kWaitNsAfterFault;
         if (g.n1 + g.n2 > 0) {
           // kRows / HPU rows of each stacked head (an absent head repeats the last one;
           // its rows are masked)
           const int qrow = g.l * la.sum_text + g.x0;
-          ptx::mbar_arrive_expect_tx(q_full, 2u * q_half);
+          ptx::mbar_arrive_expect_tx(q_full + qb, 2u * q_half);
 #pragma unroll
           for (int hs = 0; hs < (SPLIT ? 2 : HPU); ++hs) {
             const int hq = SPLIT ? g.h : g.h + min(hs, g.nh - 1);
             const uint32_t off = (uint32_t)(hs * (SPLIT ? kRows / 2 : kRph)) * 128u;
-            ptx::tma_load_3d(q_sm + off, &tmQ, q_full, 0, hq, qrow);
-            ptx::tma_load_3d(q_sm + q_half + off, &tmQ, q_full, 64, hq, qrow);
+            ptx::tma_load_3d(q_dst + off, &tmQ, q_full + qb, 0, hq, qrow);
+            ptx::tma_load_3d(q_dst + q_half + off, &tmQ, q_full + qb, 64, hq, qrow);
           }
         } else {
-          ptx::mbar_arrive(q_full);
+          ptx::mbar_arrive(q_full + qb);
         }
         // sweep-1 tiles, then (except in a batch unit, whose visual tiles stay
         // in the ring) the visual tiles again for sweep 2
@@ -437,7 +445,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int mid = warp == 1 ? 0 : 1;
     if (lane == 0) {
       const uint32_t idesc1 = ptx::idesc_bf16_f32(kRows, kTileKeys);
-      const uint32_t q_base = ptx::smem_addr(q_sm);
       int tc = 0, u = 0, bu = 0;
       int slot = 0;          // ring stage of the next tile to consume
       uint32_t kph = 0u;     // its k_full phase
@@ -460,7 +467,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const SGeo g = stream_geo<HPU, SPLIT>(p, unit);
         const int n2c = sweep2_cols<HPU>(g.NT);
         const uint32_t idesc2 = ptx::idesc_bf16_f32(kTileKeys, n2c);
-        if (!ptx::mbar_wait(q_full, u & 1, limit, p.status)) limit = kWaitNsAfterFault;
+        const int qb = u % p.qbufs;
+        const uint32_t q_base = ptx::smem_addr(q_sm + qb * kTileBytes);
+        if (!ptx::mbar_wait(q_full + qb, (u / p.qbufs) & 1, limit, p.status))
+          limit = kWaitNsAfterFault;
         const int slot_vis = (slot + g.n_st) % p.stages;   // a batch unit's first visual tile
         for (int j = 0; j < g.n1 + (g.batch ? 0 : g.n2); ++j, ++tc) {
           const int s = slot, buf = tc & 1;
@@ -504,7 +514,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
         }
-        ptx::mma_commit(q_empty);   // every MMA of this issuer in the unit is done with Q
+        ptx::mma_commit(q_empty + qb);   // every MMA of this issuer in the unit is done with Q
         if (g.batch) {   // the next unit's accumulators wait for the batch to be read
           if (!ptx::mbar_wait(b_done, bu & 1, limit, p.status)) limit = kWaitNsAfterFault;
           ++bu;
@@ -781,19 +791,20 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-// K ring stages that fit the device's shared memory (0 if fewer than two).
-static int stream_stages() {
+// K ring stages that fit the device's shared memory beside qbufs query
+// buffers (0 if fewer than two).
+static int stream_stages(int qbufs) {
   int dev = 0, optin = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
   cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
   for (int st = kMaxStages; st >= 2; --st)
-    if ((int)(stream_plan(st, true).total + 1024) <= optin) return st;
+    if ((int)(stream_plan(st, true, qbufs).total + 1024) <= optin) return st;
   return 0;
 }
 
 // Whether the streaming kernel can take this launch: at most 128 text rows.
 bool score_stream_fits(const LayoutArgs& la) {
-  return la.max_text <= kRows && la.H % la.H_kv == 0 && stream_stages() >= 2;
+  return la.max_text <= kRows && la.H % la.H_kv == 0 && stream_stages(1) >= 2;
 }
 
 cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
@@ -809,7 +820,14 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
   // text rows leave room (64 rows: two heads, 32 rows: four)
   int hpu = 1;
   while (hpu < 4 && hpu * 2 <= p.group && la.max_text <= kRows / (hpu * 2)) hpu *= 2;
-  p.stages = stream_stages();
+  // Short units (under 24 key tiles on average) take a second query buffer,
+  // so that the next unit's first MMAs need not wait for its queries (LLaVA
+  // batch 32: 188 -> 177 us), at the cost of a K ring stage; long units keep
+  // the stage (high-resolution batch 8: 270 us with one buffer, 273 with two).
+  const long long avg_tiles =
+      ((long long)la.sum_T + la.sum_vis) / ((long long)std::max(la.B, 1) * kTileKeys);
+  p.qbufs = avg_tiles < 24 ? 2 : 1;
+  p.stages = stream_stages(p.qbufs);
   p.upk = (p.group + hpu - 1) / hpu;
   p.num_units = la.B * la.L * la.H_kv * p.upk;
   p.scale = 1.0f / sqrtf(128.0f);
@@ -838,7 +856,7 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
       !make_score_map(&tmK, k, la.H_kv, (int64_t)la.L * la.sum_T, k_stride, kTileKeys))
     return cudaErrorInvalidValue;
   if (p.stages < 2) return cudaErrorInvalidValue;
-  const size_t smem = stream_plan(p.stages, p.sched != nullptr).total + 1024;
+  const size_t smem = stream_plan(p.stages, p.sched != nullptr, p.qbufs).total + 1024;
   const dim3 grid((unsigned)grid_n);
   const bool dyn = p.sched != nullptr;
   auto go = [&](auto kernel) {
