@@ -124,7 +124,7 @@ constexpr int kURing = 4;        // unit indices in flight from the producer to 
 constexpr int kOrderMax = 256;   // images the heaviest-first order covers
 
 struct SPlan {
-  uint32_t q, k, bars, slot, ms, lse, cps, red, ring, order, cost, ubars, total;
+  uint32_t q, k, bars, slot, ms, lse, cps, red, imgs, ring, order, cost, ubars, total;
 };
 
 // dyn: with the unit ring, its barriers and the image order (round-robin
@@ -139,7 +139,8 @@ __host__ __device__ inline SPlan stream_plan(int stages, bool dyn, int qbufs) {
   s.lse = s.ms + 4u * kRows * 8u;                       // [128] float -lse per text row
   s.cps = s.lse + kRows * 4u;                           // [2][8 chunks][128 keys] partials
   s.red = s.cps + 2u * 8u * kTileKeys * 4u;             // [4 heads][4] float4 statistics
-  s.ring = s.red + 16u * 16u;                           // [kURing] int unit indices
+  s.imgs = s.red + 16u * 16u;                           // [kOrderMax] SImg image layouts
+  s.ring = s.imgs + 32u * kOrderMax;                    // [kURing] int unit indices
   s.order = s.ring + 4u * kURing;                       // [kOrderMax] int images, heaviest first
   s.cost = s.order + 4u * kOrderMax;                    // [kOrderMax] float image costs
   s.ubars = s.cost + 4u * kOrderMax;                    // [2][kURing] unit-ring mbarriers
@@ -167,8 +168,36 @@ struct SGeo {
   bool ok, batch;
 };
 
+// One image's layout as the units need it, staged per CTA in shared memory:
+// S, N_V, N_T, first token, first text row, first visual row, and whether
+// the layout arrays are consistent for it (the checks of stream_geo).
+struct SImg {
+  int S, NV, NT, t0, x0, v0, ok, pad;
+};
+
+template <bool SPLIT, int HPU>
+__device__ __forceinline__ SImg load_image(const LayoutArgs& la, int b) {
+  SImg m;
+  m.S = __ldg(la.n_sys + b);
+  m.NV = __ldg(la.n_vis + b);
+  m.NT = __ldg(la.n_text + b);
+  m.t0 = __ldg(la.tok_off + b);
+  m.x0 = __ldg(la.text_off + b);
+  m.v0 = __ldg(la.vis_off + b);
+  const int T = m.S + m.NV + m.NT;
+  m.ok = m.S >= 0 && m.NV >= 0 && m.NT >= 1 && m.NT <= (SPLIT ? kRows / 2 : kRows / HPU) &&
+         T <= la.max_T && m.NV <= la.max_vis && __ldg(la.tok_off + b + 1) - m.t0 == T &&
+         m.t0 >= 0 && m.t0 + T <= la.sum_T && __ldg(la.text_off + b + 1) - m.x0 == m.NT &&
+         m.x0 >= 0 && m.x0 + m.NT <= la.sum_text && __ldg(la.vis_off + b + 1) - m.v0 == m.NV &&
+         m.v0 >= 0 && m.v0 + m.NV <= la.sum_vis;
+  m.pad = 0;
+  return m;
+}
+
+// imgs: the images' layouts in shared memory (la.B <= kOrderMax), or null
+// to read them from global memory.
 template <int HPU, bool SPLIT>
-__device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit) {
+__device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit, const SImg* imgs) {
   const LayoutArgs& la = p.la;
   SGeo g;
   if (HPU == 1) {   // units are (image, layer, query head)
@@ -185,18 +214,15 @@ __device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit) {
     g.h = g.kvh * p.group + ug * HPU;
     g.nh = min(HPU, p.group - ug * HPU);
   }
-  g.S = __ldg(la.n_sys + g.b);
-  g.NV = __ldg(la.n_vis + g.b);
-  g.NT = __ldg(la.n_text + g.b);
-  g.t0 = __ldg(la.tok_off + g.b);
-  g.x0 = __ldg(la.text_off + g.b);
-  g.v0 = __ldg(la.vis_off + g.b);
+  const SImg m = imgs ? imgs[g.b] : load_image<SPLIT, HPU>(la, g.b);
+  g.S = m.S;
+  g.NV = m.NV;
+  g.NT = m.NT;
+  g.t0 = m.t0;
+  g.x0 = m.x0;
+  g.v0 = m.v0;
   const int T = g.S + g.NV + g.NT;
-  g.ok = g.S >= 0 && g.NV >= 0 && g.NT >= 1 && g.NT <= (SPLIT ? kRows / 2 : kRows / HPU) && T <= la.max_T &&
-         g.NV <= la.max_vis && __ldg(la.tok_off + g.b + 1) - g.t0 == T && g.t0 >= 0 &&
-         g.t0 + T <= la.sum_T && __ldg(la.text_off + g.b + 1) - g.x0 == g.NT && g.x0 >= 0 &&
-         g.x0 + g.NT <= la.sum_text && __ldg(la.vis_off + g.b + 1) - g.v0 == g.NV &&
-         g.v0 >= 0 && g.v0 + g.NV <= la.sum_vis;
+  g.ok = m.ok != 0;
   const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
   g.n2 = g.ok ? (g.NV + kTileKeys - 1) / kTileKeys : 0;
   g.n_st = (g.S + kTileKeys - 1) / kTileKeys;
@@ -261,6 +287,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* uring = reinterpret_cast<volatile int*>(smem + plan.ring);
   int* order_s = reinterpret_cast<int*>(smem + plan.order);
   float* cost_s = reinterpret_cast<float*>(smem + plan.cost);
+  SImg* imgs_s = reinterpret_cast<SImg*>(smem + plan.imgs);
+  const SImg* imgs = la.B <= kOrderMax ? imgs_s : nullptr;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + plan.slot);
   float2* ms = reinterpret_cast<float2*>(smem + plan.ms);
   float* nlse = reinterpret_cast<float*>(smem + plan.lse);   // -lse per text row
@@ -301,6 +329,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     ptx::prefetch_tensormap(&tmK);
   }
   if (warp == 1) ptx::tmem_alloc(tmem_slot, kTmemCols);
+  // every image's layout into shared memory once (the barrier below publishes
+  // it), so that a unit's geometry is not a chain of global loads at its start
+  if (imgs)
+    for (int i = threadIdx.x; i < la.B; i += blockDim.x) imgs_s[i] = load_image<SPLIT, HPU>(la, i);
   if (DYN && p.order) {
     // Every CTA derives the same order.  With few units per CTA (order 2)
     // or when the costliest image costs more than twice the mean, images go
@@ -371,7 +403,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int ld = 0;
       int unit = publish(0, (int)blockIdx.x);   // the CTA's own first unit
       for (int u = 0; unit >= 0; ++u) {
-        const SGeo g = stream_geo<HPU, SPLIT>(p, unit);
+        const SGeo g = stream_geo<HPU, SPLIT>(p, unit, imgs);
         if (!g.ok) E2S_DEV_FLAG(p.status, E2S_ERR_SHAPE);
         // unit u's queries go into buffer u % qbufs once the unit qbufs back is
         // done with it (with two, they land while the previous unit finishes)
@@ -416,7 +448,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                             : (int)blockIdx.x + (u + 1) * (int)gridDim.x);
         unit = next;
         if (next >= 0) {
-          const SGeo gn = stream_geo<HPU, SPLIT>(p, next);
+          const SGeo gn = stream_geo<HPU, SPLIT>(p, next, imgs);
           if (gn.n1 + gn.n2 > 0) {
             const int qrow = gn.l * la.sum_text + gn.x0;
 #pragma unroll
@@ -464,7 +496,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (;; ++u) {
         const int unit = take_unit(u, false);
         if (unit < 0) break;
-        const SGeo g = stream_geo<HPU, SPLIT>(p, unit);
+        const SGeo g = stream_geo<HPU, SPLIT>(p, unit, imgs);
         const int n2c = sweep2_cols<HPU>(g.NT);
         const uint32_t idesc2 = ptx::idesc_bf16_f32(kTileKeys, n2c);
         const int qb = u % p.qbufs;
@@ -533,7 +565,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int u = 0;; ++u) {
       const int unit = take_unit(u, true);
       if (unit < 0) break;
-      const SGeo g = stream_geo<HPU, SPLIT>(p, unit);
+      const SGeo g = stream_geo<HPU, SPLIT>(p, unit, imgs);
       // TMEM row lrow holds text row t of stacked head hs (SPLIT: row lrow % 64)
       const int hs = SPLIT ? 0 : lrow / kRph;
       const int t = SPLIT ? (lrow & (kRows / 2 - 1)) : lrow - hs * kRph;
