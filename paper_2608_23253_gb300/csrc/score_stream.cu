@@ -116,6 +116,8 @@ struct StreamArgs {
   uint32_t* sched;      // nullable: [0] units handed out after the first, [1] CTAs done
   int upi;              // units per image
   int qbufs;            // query buffers: 2 lets the next unit's queries land early
+  int rsplit;           // one head per unit, not SPLIT: units of <= 64 text rows run split
+                        // (the query map's box is then 64 rows)
   int order;            // 0: index order; 1: heaviest first if the costs are skewed;
                         // 2: heaviest first (la.B <= kOrderMax)
 };
@@ -166,6 +168,7 @@ struct SGeo {
   // sweep 2 issues all its MMAs at once from there.
   int n_st, n_tt, kfirst;
   bool ok, batch;
+  bool sp;   // split rows: the unit's <= 64 text rows fill lanes 0-63 and again 64-127
 };
 
 // One image's layout as the units need it, staged per CTA in shared memory:
@@ -229,6 +232,7 @@ __device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit, const 
   g.n_tt = max(0, (g.NV + g.NT + kTileKeys - 1) / kTileKeys - g.n2);
   // with the rows' lse given (from the layer's attention pass) there is no sweep 1
   const bool given = p.lse_in != nullptr;
+  g.sp = SPLIT || (HPU == 1 && p.rsplit && g.NT <= kRows / 2);
   g.batch = !given && HPU == 1 && g.ok && causal && g.n2 >= 1 && g.n2 <= kMaxBatch &&
             g.n2 * sweep2_cols<HPU>(g.NT) <= kTmemCols && g.n2 + g.n_tt <= p.stages;
   g.kfirst = g.batch ? g.S - kTileKeys * g.n_st : 0;
@@ -413,15 +417,18 @@ __global__ void __launch_bounds__(kThreads, 1)
           limit = kWaitNsAfterFault;
         if (g.n1 + g.n2 > 0) {
           // kRows / HPU rows of each stacked head (an absent head repeats the last one;
-          // its rows are masked)
+          // its rows are masked); with 64-row boxes (one head) two boxes: the
+          // unit's first 64 rows twice when it runs split, else rows 0-63 and 64-127
           const int qrow = g.l * la.sum_text + g.x0;
+          const bool box64 = SPLIT || (HPU == 1 && p.rsplit);
           ptx::mbar_arrive_expect_tx(q_full + qb, 2u * q_half);
 #pragma unroll
-          for (int hs = 0; hs < (SPLIT ? 2 : HPU); ++hs) {
-            const int hq = SPLIT ? g.h : g.h + min(hs, g.nh - 1);
-            const uint32_t off = (uint32_t)(hs * (SPLIT ? kRows / 2 : kRph)) * 128u;
-            ptx::tma_load_3d(q_dst + off, &tmQ, q_full + qb, 0, hq, qrow);
-            ptx::tma_load_3d(q_dst + q_half + off, &tmQ, q_full + qb, 64, hq, qrow);
+          for (int hs = 0; hs < (box64 ? 2 : HPU); ++hs) {
+            const int hq = box64 ? g.h : g.h + min(hs, g.nh - 1);
+            const int row = qrow + (box64 && !g.sp ? hs * (kRows / 2) : 0);
+            const uint32_t off = (uint32_t)(hs * (box64 ? kRows / 2 : kRph)) * 128u;
+            ptx::tma_load_3d(q_dst + off, &tmQ, q_full + qb, 0, hq, row);
+            ptx::tma_load_3d(q_dst + q_half + off, &tmQ, q_full + qb, 64, hq, row);
           }
         } else {
           ptx::mbar_arrive(q_full + qb);
@@ -452,10 +459,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (gn.n1 + gn.n2 > 0) {
             const int qrow = gn.l * la.sum_text + gn.x0;
 #pragma unroll
-            for (int hs = 0; hs < (SPLIT ? 1 : HPU); ++hs) {
+            for (int hs = 0; hs < (gn.sp ? 1 : HPU == 1 && p.rsplit ? 2 : HPU); ++hs) {
               const int hq = gn.h + min(hs, gn.nh - 1);
-              ptx::tma_prefetch_3d(&tmQ, 0, hq, qrow);
-              ptx::tma_prefetch_3d(&tmQ, 64, hq, qrow);
+              const int row = qrow + (HPU == 1 && p.rsplit ? hs * (kRows / 2) : 0);
+              ptx::tma_prefetch_3d(&tmQ, 0, hq, row);
+              ptx::tma_prefetch_3d(&tmQ, 64, hq, row);
             }
             const int nt = min(gn.n1 + gn.n2, p.stages);
             for (int j = 0; j < nt; ++j) {
@@ -566,11 +574,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int unit = take_unit(u, true);
       if (unit < 0) break;
       const SGeo g = stream_geo<HPU, SPLIT>(p, unit, imgs);
-      // TMEM row lrow holds text row t of stacked head hs (SPLIT: row lrow % 64)
-      const int hs = SPLIT ? 0 : lrow / kRph;
-      const int t = SPLIT ? (lrow & (kRows / 2 - 1)) : lrow - hs * kRph;
+      // TMEM row lrow holds text row t of stacked head hs (split: row lrow % 64)
+      const bool sp = g.sp;
+      const int hs = sp ? 0 : lrow / kRph;
+      const int t = sp ? (lrow & (kRows / 2 - 1)) : lrow - hs * kRph;
       const bool rows_live =
-          hs < g.nh && (SPLIT ? (q4 & 1) * 32 : (q4 * 32) % kRph) < g.NT;   // warp-uniform
+          hs < g.nh && (sp ? (q4 & 1) * 32 : (q4 * 32) % kRph) < g.NT;   // warp-uniform
       const bool tvalid = hs < g.nh && t < g.NT;
       const int lim = tvalid ? g.S + g.NV + t : -1;   // last key this row sees
       const float inv_nt = 1.f / (float)max(g.NT, 1);
@@ -583,10 +592,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tc_fence_after();
         if (rows_live) {
 #pragma unroll
-          for (int ch = 0; ch < (SPLIT ? 1 : 2); ++ch) {
+          for (int ch = 0; ch < (sp ? 1 : 2); ++ch) {
             // 16-column chunks of this warp: 2 of its column group's 32, or
-            // (SPLIT) 1 of the 64 columns of its lane half
-            const int c16 = SPLIT ? (q4 >> 1) * (kTileKeys / 2) + cg * 16 : cg * 32 + ch * 16;
+            // (split) 1 of the 64 columns of its lane half
+            const int c16 = sp ? (q4 >> 1) * (kTileKeys / 2) + cg * 16 : cg * 32 + ch * 16;
             const int key0 = g.kfirst + kTileKeys * j + c16;
             float x[16];
             ptx::tmem_ld16(tmem + lane_base + (uint32_t)(buf * kTileKeys + c16), x);
@@ -626,7 +635,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---- merge the four column groups: lse per row (log2 domain), published
       // per text row for sweep 2 (or taken from the caller's attention pass)
       if (causal && p.lse_in != nullptr) {
-        if (cg == 0 && (!SPLIT || lrow < kRows / 2))
+        if (cg == 0 && (!sp || lrow < kRows / 2))
           nlse[lrow] = tvalid ? -__ldg(p.lse_in + ((size_t)g.l * la.H + g.h + hs) * la.sum_text +
                                        g.x0 + t) * kLog2e
                               : -kNegBig;
@@ -634,21 +643,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       } else if (causal) {
         ms[cg * kRows + lrow] = make_float2(m, ssum);
         ptx::named_bar(1, kEpiThreads);
-        // partials of this row: four column groups (and, SPLIT, both lane halves)
-        constexpr int kParts = SPLIT ? 8 : 4;
+        // partials of this row: four column groups (and, split, both lane halves)
+        const int nparts = sp ? 8 : 4;
         auto part = [&](int c) {
           return ms[(c & 3) * kRows + (c < 4 ? lrow : (lrow ^ (kRows / 2)))];
         };
         float M = kNegBig;
 #pragma unroll
-        for (int c = 0; c < kParts; ++c) M = fmaxf(M, part(c).x);
+        for (int c = 0; c < nparts; ++c) M = fmaxf(M, part(c).x);
         float L = 0.f;
 #pragma unroll
-        for (int c = 0; c < kParts; ++c) {
+        for (int c = 0; c < nparts; ++c) {
           const float2 v = part(c);
           L += v.y * fast_ex2(v.x - M);
         }
-        if (cg == 0 && (!SPLIT || lrow < kRows / 2))
+        if (cg == 0 && (!sp || lrow < kRows / 2))
           nlse[lrow] = L > 0.f ? -(M + __log2f(L)) : -kNegBig;
         ptx::named_bar(1, kEpiThreads);
       }
@@ -883,8 +892,12 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
   CUtensorMap tmQ, tmK;
   // one head of at most 64 text rows: the queries are loaded twice (SPLIT)
   const bool split = hpu == 1 && la.max_text <= kRows / 2;
+  // one head per unit with longer text somewhere in the batch: the units of at
+  // most 64 rows still run split (their rows loaded twice), so that all four
+  // lane quarters share their sweep-1 exponentials
+  p.rsplit = hpu == 1 && !split ? 1 : 0;
   if (!make_score_map(&tmQ, q, la.H, (int64_t)la.L * la.sum_text, q_stride,
-                      split ? kRows / 2 : kRows / hpu) ||
+                      split || p.rsplit ? kRows / 2 : kRows / hpu) ||
       !make_score_map(&tmK, k, la.H_kv, (int64_t)la.L * la.sum_T, k_stride, kTileKeys))
     return cudaErrorInvalidValue;
   if (p.stages < 2) return cudaErrorInvalidValue;
