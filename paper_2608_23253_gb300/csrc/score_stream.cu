@@ -117,7 +117,7 @@ struct StreamArgs {
   int upi;              // units per image
   int qbufs;            // query buffers: 2 lets the next unit's queries land early
   int rsplit;           // one head per unit, not SPLIT: units of <= 64 text rows run split
-                        // (the query map's box is then 64 rows)
+                        // (the query map's box is then 64 rows; the RS kernels)
   int order;            // 0: index order; 1: heaviest first if the costs are skewed;
                         // 2: heaviest first (la.B <= kOrderMax)
 };
@@ -199,7 +199,7 @@ __device__ __forceinline__ SImg load_image(const LayoutArgs& la, int b) {
 
 // imgs: the images' layouts in shared memory (la.B <= kOrderMax), or null
 // to read them from global memory.
-template <int HPU, bool SPLIT>
+template <int HPU, bool SPLIT, bool RS>
 __device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit, const SImg* imgs) {
   const LayoutArgs& la = p.la;
   SGeo g;
@@ -232,7 +232,7 @@ __device__ __forceinline__ SGeo stream_geo(const StreamArgs& p, int unit, const 
   g.n_tt = max(0, (g.NV + g.NT + kTileKeys - 1) / kTileKeys - g.n2);
   // with the rows' lse given (from the layer's attention pass) there is no sweep 1
   const bool given = p.lse_in != nullptr;
-  g.sp = SPLIT || (HPU == 1 && p.rsplit && g.NT <= kRows / 2);
+  g.sp = SPLIT || (RS && HPU == 1 && g.NT <= kRows / 2);
   g.batch = !given && HPU == 1 && g.ok && causal && g.n2 >= 1 && g.n2 <= kMaxBatch &&
             g.n2 * sweep2_cols<HPU>(g.NT) <= kTmemCols && g.n2 + g.n_tt <= p.stages;
   g.kfirst = g.batch ? g.S - kTileKeys * g.n_st : 0;
@@ -263,9 +263,11 @@ __device__ __forceinline__ int unit_of(const StreamArgs& p, const int* order, in
 // most 64 text rows): the queries fill TMEM lanes 0-63 and again 64-127, and
 // in sweep 1 each half of the lanes takes half of every key tile's columns, so
 // all four lane quarters (all four SM sub-partitions) share the exponentials.
-// DYN: units come from the workspace counter through the unit ring (p.sched
-// set); otherwise round-robin, and the ring's code is compiled out.
-template <int HPU, bool SPLIT, bool DYN>
+// RS (one head, not SPLIT): units of at most 64 text rows run split, the
+// others not (p.rsplit; the query map's box is 64 rows).  DYN: units come
+// from the workspace counter through the unit ring (p.sched set); otherwise
+// round-robin, and the ring's code is compiled out.
+template <int HPU, bool SPLIT, bool RS, bool DYN>
 __global__ void __launch_bounds__(kThreads, 1)
     score_stream_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmK, const StreamArgs p) {
@@ -407,7 +409,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int ld = 0;
       int unit = publish(0, (int)blockIdx.x);   // the CTA's own first unit
       for (int u = 0; unit >= 0; ++u) {
-        const SGeo g = stream_geo<HPU, SPLIT>(p, unit, imgs);
+        const SGeo g = stream_geo<HPU, SPLIT, RS>(p, unit, imgs);
         if (!g.ok) E2S_DEV_FLAG(p.status, E2S_ERR_SHAPE);
         // unit u's queries go into buffer u % qbufs once the unit qbufs back is
         // done with it (with two, they land while the previous unit finishes)
@@ -420,7 +422,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // its rows are masked); with 64-row boxes (one head) two boxes: the
           // unit's first 64 rows twice when it runs split, else rows 0-63 and 64-127
           const int qrow = g.l * la.sum_text + g.x0;
-          const bool box64 = SPLIT || (HPU == 1 && p.rsplit);
+          constexpr bool box64 = SPLIT || RS;
           ptx::mbar_arrive_expect_tx(q_full + qb, 2u * q_half);
 #pragma unroll
           for (int hs = 0; hs < (box64 ? 2 : HPU); ++hs) {
@@ -455,13 +457,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                                             : (int)blockIdx.x + (u + 1) * (int)gridDim.x);
         unit = next;
         if (next >= 0) {
-          const SGeo gn = stream_geo<HPU, SPLIT>(p, next, imgs);
+          const SGeo gn = stream_geo<HPU, SPLIT, RS>(p, next, imgs);
           if (gn.n1 + gn.n2 > 0) {
             const int qrow = gn.l * la.sum_text + gn.x0;
 #pragma unroll
-            for (int hs = 0; hs < (gn.sp ? 1 : HPU == 1 && p.rsplit ? 2 : HPU); ++hs) {
+            for (int hs = 0; hs < (gn.sp ? 1 : RS ? 2 : HPU); ++hs) {
               const int hq = gn.h + min(hs, gn.nh - 1);
-              const int row = qrow + (HPU == 1 && p.rsplit ? hs * (kRows / 2) : 0);
+              const int row = qrow + (RS ? hs * (kRows / 2) : 0);
               ptx::tma_prefetch_3d(&tmQ, 0, hq, row);
               ptx::tma_prefetch_3d(&tmQ, 64, hq, row);
             }
@@ -504,7 +506,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (;; ++u) {
         const int unit = take_unit(u, false);
         if (unit < 0) break;
-        const SGeo g = stream_geo<HPU, SPLIT>(p, unit, imgs);
+        const SGeo g = stream_geo<HPU, SPLIT, RS>(p, unit, imgs);
         const int n2c = sweep2_cols<HPU>(g.NT);
         const uint32_t idesc2 = ptx::idesc_bf16_f32(kTileKeys, n2c);
         const int qb = u % p.qbufs;
@@ -573,7 +575,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int u = 0;; ++u) {
       const int unit = take_unit(u, true);
       if (unit < 0) break;
-      const SGeo g = stream_geo<HPU, SPLIT>(p, unit, imgs);
+      const SGeo g = stream_geo<HPU, SPLIT, RS>(p, unit, imgs);
       // TMEM row lrow holds text row t of stacked head hs (split: row lrow % 64)
       const bool sp = g.sp;
       const int hs = sp ? 0 : lrow / kRph;
@@ -894,8 +896,10 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
   const bool split = hpu == 1 && la.max_text <= kRows / 2;
   // one head per unit with longer text somewhere in the batch: the units of at
   // most 64 rows still run split (their rows loaded twice), so that all four
-  // lane quarters share their sweep-1 exponentials
-  p.rsplit = hpu == 1 && !split ? 1 : 0;
+  // lane quarters share their sweep-1 exponentials -- when the text is short
+  // on average (below 96 rows); a batch of long text only pays the branches
+  // (high-resolution batch 8: +1.5 %)
+  p.rsplit = hpu == 1 && !split && la.sum_text < (long long)la.B * 96 ? 1 : 0;
   if (!make_score_map(&tmQ, q, la.H, (int64_t)la.L * la.sum_text, q_stride,
                       split || p.rsplit ? kRows / 2 : kRows / hpu) ||
       !make_score_map(&tmK, k, la.H_kv, (int64_t)la.L * la.sum_T, k_stride, kTileKeys))
@@ -908,12 +912,19 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
     return launch_kernel(kernel, grid, dim3(kThreads), smem, st, 0, false, tmQ, tmK, p);
   };
   if (hpu == 4)
-    return dyn ? go(score_stream_kernel<4, false, true>) : go(score_stream_kernel<4, false, false>);
+    return dyn ? go(score_stream_kernel<4, false, false, true>)
+               : go(score_stream_kernel<4, false, false, false>);
   if (hpu == 2)
-    return dyn ? go(score_stream_kernel<2, false, true>) : go(score_stream_kernel<2, false, false>);
+    return dyn ? go(score_stream_kernel<2, false, false, true>)
+               : go(score_stream_kernel<2, false, false, false>);
   if (split)
-    return dyn ? go(score_stream_kernel<1, true, true>) : go(score_stream_kernel<1, true, false>);
-  return dyn ? go(score_stream_kernel<1, false, true>) : go(score_stream_kernel<1, false, false>);
+    return dyn ? go(score_stream_kernel<1, true, false, true>)
+               : go(score_stream_kernel<1, true, false, false>);
+  if (p.rsplit)
+    return dyn ? go(score_stream_kernel<1, false, true, true>)
+               : go(score_stream_kernel<1, false, true, false>);
+  return dyn ? go(score_stream_kernel<1, false, false, true>)
+             : go(score_stream_kernel<1, false, false, false>);
 }
 
 }  // namespace e2s
