@@ -93,12 +93,12 @@ STREAM_SOURCES = ("score_stream.cu", "sm100_ptx.cuh", "device_common.cuh")
 NCU_TENSOR_PIPE = {
     "cfg1": {"kernel": "score_split_kernel", "src": KERNEL_SOURCES, "sha": "70b211816da11f00",
              "pct": 15.71, "profile": "profiles/score_split_kernel_llava_b1.md"},
-    "cfg2": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "f47ead7b3205110f",
-             "pct": 25.00, "profile": "profiles/score_stream_kernel_llava_b32.md"},
-    "cfg3": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "f47ead7b3205110f",
-             "pct": 31.91, "profile": "profiles/score_stream_kernel_qwen2vl_b16.md"},
-    "cfg4": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "f47ead7b3205110f",
-             "pct": 36.77, "profile": "profiles/score_stream_kernel_highres_b8.md"},
+    "cfg2": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "a05d629d649c0906",
+             "pct": 26.76, "profile": "profiles/score_stream_kernel_llava_b32.md"},
+    "cfg3": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "a05d629d649c0906",
+             "pct": 31.66, "profile": "profiles/score_stream_kernel_qwen2vl_b16.md"},
+    "cfg4": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "a05d629d649c0906",
+             "pct": 36.57, "profile": "profiles/score_stream_kernel_highres_b8.md"},
 }
 
 
