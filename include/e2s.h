@@ -345,6 +345,12 @@ e2s_status e2s_select(const e2s_layout* layout, const e2s_params* params,
  *   src[i], dst[i]  n_tensors (1..32) HOST arrays of DEVICE pointers to
  *                   row-major [sum_T][row] and [sum_T - sum_vis + sum_keep][row]
  *                   tensors (e.g. hidden states and each layer's K and V).
+ *                   A source may also be page-locked host memory the device
+ *                   can address (cudaHostAlloc, or cudaHostRegister with
+ *                   mapping, under unified addressing): the kernel then reads
+ *                   only the rows it keeps across the host link.  (e2s_prune
+ *                   prefetches every candidate row into L2: give it device
+ *                   sources.)
  *   row_bytes[i]    HOST array; each a positive multiple of 16; pointers
  *                   16-byte aligned.
  *   pos_ids_out     nullable int32 [total rows]: image-local original position
