@@ -84,6 +84,35 @@ def test_compaction_bit_exact(keep):
     assert R == 35 + keep + 64
 
 
+def test_compaction_from_pinned_host_sources():
+    """e2s_compact with the hidden states and V in page-locked host memory (read
+    in place across the host link) gathers the oracle's rows bit-exactly, on a
+    ragged batch, beside K from device memory."""
+    dev = device()
+    inp = config_inputs(2, 6, None, True)
+    ref = orc.decide(inp.q_text, inp.k, inp.n_sys, inp.n_vis, inp.n_text, inp.grid_h, inp.grid_w,
+                     inp.keep, H_kv=inp.spec.H_kv, params=orc.Params())
+    gpu = run_gpu(inp, "causal")
+    dec = gpu["decision"]
+    dec.keep_idx.copy_(torch.as_tensor(np.concatenate(ref["keep"]).astype(np.int32), device=dev))
+    from paper_2608_23253_gb300.decision import bf16_tensor
+    L, T = inp.spec.L, inp.k.shape[1]
+    host = [inp.hidden] + [inp.k[l].reshape(T, -1) for l in range(L)] + \
+           [inp.v[l].reshape(T, -1) for l in range(L)]
+    pinned = lambda x: torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).pin_memory()  # noqa: E731
+    src = [pinned(host[0])] + [bf16_tensor(h, dev) for h in host[1:1 + L]] + \
+          [pinned(h) for h in host[1 + L:]]
+    R = dec.out_rows()
+    dst = [torch.empty((R, t.shape[1]), dtype=torch.bfloat16, device=dev) for t in src]
+    pos = torch.empty(R, dtype=torch.int32, device=dev)
+    dec.compact(src, dst, pos)
+    torch.cuda.synchronize()
+    assert dec.status() == 0
+    for d_, h_ in zip(dst, host):
+        want = orc.compact(h_, inp.n_sys, inp.n_vis, inp.n_text, ref["keep"])
+        assert np.array_equal(d_.cpu().view(torch.int16).numpy().view(np.uint16), want)
+
+
 def test_ragged_compaction_bit_exact():
     dev = device()
     inp = config_inputs(2, 6, None, True)
