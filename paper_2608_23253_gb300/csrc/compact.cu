@@ -169,7 +169,6 @@ __global__ void __launch_bounds__(kCompactThreads)
                    int early, int prefetch) {
   __shared__ ImgRows tab_s[kTabImages];
   const ImgRows* tab = la.B <= kTabImages ? tab_s : nullptr;
-  pdl_launch_dependents();
   if (early) {
     if (prefetch) prefetch_visual_rows(la, n_tensors, ts);
     if (tab) stage_images(la, keep_off, tab_s);
@@ -184,6 +183,9 @@ __global__ void __launch_bounds__(kCompactThreads)
     compact_rows<RV>(la, keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, -1, false,
                  tab);
   }
+  // the next kernel may be scheduled once this one is finishing (signalled
+  // earlier, its CTAs would hold SMs while the copies run)
+  pdl_launch_dependents();
 }
 
 }  // namespace

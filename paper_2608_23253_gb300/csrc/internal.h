@@ -76,7 +76,7 @@ inline LayoutArgs layout_args(const e2s_layout* l) {
 cudaError_t launch_score_tc(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                             const void* k, int64_t k_stride, float* a_out, float4* stats,
                             uint32_t* counters, uint32_t* status, cudaStream_t st,
-                            int* unsupported);
+                            int* unsupported, bool pdl = false);
 // Streaming score kernel (long sequences, GQA; at most 128 text rows).  With
 // lse_in (natural-log lse of every text row, [L][H][sum_text]) it skips the
 // normaliser sweep and streams only the visual key tiles.
@@ -84,7 +84,7 @@ bool score_stream_fits(const LayoutArgs& la);
 cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                                 const void* k, int64_t k_stride, float* a_out, float4* stats,
                                 uint32_t* counters, uint32_t* status, cudaStream_t st,
-                                const float* lse_in = nullptr);
+                                const float* lse_in = nullptr, bool pdl = false);
 // Cluster-per-unit score kernel for small batches (key tiles split over the
 // cluster's CTAs): its cluster size and tiles per CTA, or false when it does
 // not take the launch.  lse_in as for launch_score_stream.
@@ -92,7 +92,7 @@ bool score_split_plan(const LayoutArgs& la, int mode, bool lse, int* cluster, in
 cudaError_t launch_score_split(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                                const void* k, int64_t k_stride, float* a_out, float4* stats,
                                uint32_t* counters, uint32_t* status, cudaStream_t st,
-                               const float* lse_in, int cluster, int tpc);
+                               const float* lse_in, int cluster, int tpc, bool pdl = false);
 // The pruning layer's causal attention (O and the row lse) with the text rows'
 // score a and its Eq. 8 statistics as a by-product when a_out is given.
 // sched: two workspace words, zero on entry and on return (the item counter
@@ -107,7 +107,8 @@ bool score_unit_fits(const LayoutArgs& la, int mode);
 bool score_unit_single_group(const LayoutArgs& la, int mode);
 cudaError_t launch_score_unit(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                               const void* k, int64_t k_stride, float* a_out, float4* stats,
-                              uint32_t* counters, uint32_t* status, cudaStream_t st);
+                              uint32_t* counters, uint32_t* status, cudaStream_t st,
+                              bool pdl = false);
 cudaError_t launch_score_simt(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                               const void* k, int64_t k_stride, float* a_out, float4* stats,
                               uint32_t* counters, uint32_t* status, cudaStream_t st);

@@ -196,6 +196,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
   ptx::cluster_arrive_relaxed();   // phase 0: every CTA of the cluster is running
   pdl_launch_dependents();
+  pdl_wait();   // inputs may come from the kernel before (launched with PDL)
   if (p.counters != nullptr && blockIdx.x == 0)
     for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
       p.counters[i] = 0u;
@@ -516,7 +517,7 @@ bool score_split_plan(const LayoutArgs& la, int mode, bool lse, int* cluster, in
 cudaError_t launch_score_split(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                                const void* k, int64_t k_stride, float* a_out, float4* stats,
                                uint32_t* counters, uint32_t* status, cudaStream_t st,
-                               const float* lse_in, int cluster, int tpc) {
+                               const float* lse_in, int cluster, int tpc, bool pdl) {
   SplitArgs p;
   p.la = la;
   p.mode = mode;
@@ -554,7 +555,7 @@ cudaError_t launch_score_split(const LayoutArgs& la, int mode, const void* q, in
       !make_score_map(&tmK, k, la.H_kv, (int64_t)la.L * la.sum_T, k_stride, kTileKeys))
     return cudaErrorInvalidValue;
   return launch_kernel(score_split_kernel, dim3((unsigned)(p.num_units * cluster)),
-                       dim3(kThreads), smem, st, cluster, false, tmQ, tmK, p);
+                       dim3(kThreads), smem, st, cluster, pdl, tmQ, tmK, p);
 }
 
 }  // namespace e2s

@@ -305,6 +305,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
   constexpr int kRph = kRows / HPU;   // TMEM lanes per stacked head
   pdl_launch_dependents();   // every CTA is resident: the next kernel may be scheduled
+  pdl_wait();   // inputs may come from the kernel before (launched with PDL)
   if (p.counters != nullptr && blockIdx.x == 0)
     for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
       p.counters[i] = 0u;
@@ -853,7 +854,7 @@ bool score_stream_fits(const LayoutArgs& la) {
 cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                                 const void* k, int64_t k_stride, float* a_out, float4* stats,
                                 uint32_t* counters, uint32_t* status, cudaStream_t st,
-                                const float* lse_in) {
+                                const float* lse_in, bool pdl) {
   StreamArgs p;
   p.lse_in = lse_in;
   p.la = la;
@@ -909,7 +910,7 @@ cudaError_t launch_score_stream(const LayoutArgs& la, int mode, const void* q, i
   const dim3 grid((unsigned)grid_n);
   const bool dyn = p.sched != nullptr;
   auto go = [&](auto kernel) {
-    return launch_kernel(kernel, grid, dim3(kThreads), smem, st, 0, false, tmQ, tmK, p);
+    return launch_kernel(kernel, grid, dim3(kThreads), smem, st, 0, pdl, tmQ, tmK, p);
   };
   if (hpu == 4)
     return dyn ? go(score_stream_kernel<4, false, false, true>)

@@ -144,6 +144,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   const int ncs = p.hpc * p.ntp_max;
   const uint32_t q_half = (uint32_t)ncs * 128u;
   pdl_launch_dependents();
+  pdl_wait();   // inputs may come from the kernel before (launched with PDL)
   if (p.counters != nullptr && blockIdx.x == 0)
     for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
       p.counters[i] = 0u;
@@ -502,7 +503,7 @@ bool make_score_map(CUtensorMap* map, const void* base, int heads, int64_t rows,
 cudaError_t launch_score_tc(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                             const void* k, int64_t k_stride, float* a_out, float4* stats,
                             uint32_t* counters, uint32_t* status, cudaStream_t st,
-                            int* unsupported) {
+                            int* unsupported, bool pdl) {
   *unsupported = 0;
   // kernel choice (measured): the cluster-per-unit kernel when every unit's
   // key tiles spread over at most two CTAs per SM in one wave (batch 1); the
@@ -514,17 +515,17 @@ cudaError_t launch_score_tc(const LayoutArgs& la, int mode, const void* q, int64
   int split_c = 0, split_t = 0;
   if (score_split_plan(la, mode, false, &split_c, &split_t))
     return launch_score_split(la, mode, q, q_stride, k, k_stride, a_out, stats, counters, status,
-                              st, nullptr, split_c, split_t);
+                              st, nullptr, split_c, split_t, pdl);
   const bool unit = score_unit_fits(la, mode);
   if (unit && score_unit_single_group(la, mode))
     return launch_score_unit(la, mode, q, q_stride, k, k_stride, a_out, stats, counters, status,
-                             st);
+                             st, pdl);
   if (score_stream_fits(la))
     return launch_score_stream(la, mode, q, q_stride, k, k_stride, a_out, stats, counters, status,
-                               st);
+                               st, nullptr, pdl);
   if (unit)
     return launch_score_unit(la, mode, q, q_stride, k, k_stride, a_out, stats, counters, status,
-                             st);
+                             st, pdl);
   TcArgs p;
   p.la = la;
   p.group = la.H / la.H_kv;
@@ -584,7 +585,7 @@ cudaError_t launch_score_tc(const LayoutArgs& la, int mode, const void* q, int64
     return cudaErrorInvalidValue;
   const long long units = (long long)la.B * la.L * la.H_kv * p.groups_per_kv;
   return launch_kernel(score_tc_kernel, dim3((unsigned)(units * p.cluster)), dim3(kThreads), smem,
-                       st, p.cluster, false, tmQ, tmK, p);
+                       st, p.cluster, pdl, tmQ, tmK, p);
 }
 
 }  // namespace e2s

@@ -196,6 +196,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t q_half = (uint32_t)p.ntp_max * 128u;
   const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
   pdl_launch_dependents();   // every CTA is resident: the next kernel may be scheduled
+  pdl_wait();   // inputs may come from the kernel before (launched with PDL)
   if (p.counters != nullptr && blockIdx.x == 0)
     for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
       p.counters[i] = 0u;
@@ -499,6 +500,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t q_half = (uint32_t)p.ntg * 128u;
   const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
   pdl_launch_dependents();   // every CTA is resident: the next kernel may be scheduled
+  pdl_wait();   // inputs may come from the kernel before (launched with PDL)
   if (p.counters != nullptr && blockIdx.x == 0)
     for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
       p.counters[i] = 0u;
@@ -843,7 +845,8 @@ bool score_unit_fits(const LayoutArgs& la, int mode) {
 
 cudaError_t launch_score_unit(const LayoutArgs& la, int mode, const void* q, int64_t q_stride,
                               const void* k, int64_t k_stride, float* a_out, float4* stats,
-                              uint32_t* counters, uint32_t* status, cudaStream_t st) {
+                              uint32_t* counters, uint32_t* status, cudaStream_t st,
+                              bool pdl) {
   UnitArgs p;
   p.la = la;
   p.ntp_max = ((std::max(la.max_text, 1) + 15) / 16) * 16;
@@ -864,8 +867,8 @@ cudaError_t launch_score_unit(const LayoutArgs& la, int mode, const void* q, int
   const size_t smem = unit_plan(p.ntg).total + 1024;
   const dim3 grid((unsigned)std::min(p.num_units, sm_count()));
   if (p.ntg >= p.ntp_max)
-    return launch_kernel(score_unit_kernel, grid, dim3(kThreads), smem, st, 0, false, tmQ, tmK, p);
-  return launch_kernel(score_group_kernel, grid, dim3(kThreads), smem, st, 0, false, tmQ, tmK, p);
+    return launch_kernel(score_unit_kernel, grid, dim3(kThreads), smem, st, 0, pdl, tmQ, tmK, p);
+  return launch_kernel(score_group_kernel, grid, dim3(kThreads), smem, st, 0, pdl, tmQ, tmK, p);
 }
 
 }  // namespace e2s
