@@ -76,7 +76,7 @@ WORKLOADS = {
 KERNEL_SOURCES = ("score_split.cu", "sm100_ptx.cuh", "device_common.cuh")
 NCU_TRAFFIC = {
     "cfg1": {"stage": "score", "kernel": "score_split_kernel", "src": KERNEL_SOURCES,
-             "sha": "70b211816da11f00", "bytes": 18226688},
+             "sha": "35c56e8a43f2f801", "bytes": 18227200},
 }
 
 
@@ -91,8 +91,8 @@ ABLATIONS = {"A1": ("vanilla: q = mean attention, no novelty", 16),
 # (profiles/score_*_kernel_*.md), with the source hash they were taken on.
 STREAM_SOURCES = ("score_stream.cu", "sm100_ptx.cuh", "device_common.cuh")
 NCU_TENSOR_PIPE = {
-    "cfg1": {"kernel": "score_split_kernel", "src": KERNEL_SOURCES, "sha": "70b211816da11f00",
-             "pct": 15.71, "profile": "profiles/score_split_kernel_llava_b1.md"},
+    "cfg1": {"kernel": "score_split_kernel", "src": KERNEL_SOURCES, "sha": "35c56e8a43f2f801",
+             "pct": 14.15, "profile": "profiles/score_split_kernel_llava_b1.md"},
     "cfg2": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "a05d629d649c0906",
              "pct": 26.76, "profile": "profiles/score_stream_kernel_llava_b32.md"},
     "cfg3": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "a05d629d649c0906",
