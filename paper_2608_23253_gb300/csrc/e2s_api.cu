@@ -204,8 +204,9 @@ e2s_status prune_impl(const e2s_layout* layout, const e2s_params* params,
                      mass_out, fused_out, q_out, keep_count, keep_off, sum_keep, keep_idx,
                      q_tilde_out, ws, st, lse_text, true));
   if (n_tensors == 0 && !pos_ids_out) return E2S_OK;
-  // the score kernel is an ordinary launch: it starts after all earlier work on
-  // the stream, so the sources are complete before the compaction may start
+  // the score kernel signals its dependents only after its own wait on the
+  // kernel before it, so the sources are complete before the compaction (which
+  // copies the system and text rows before its wait) may start
   return from_cuda(launch_compact(layout_args(layout), keep_idx, keep_off, sum_keep, n_tensors,
                                   src, dst, row_bytes, pos_ids_out, status_word(ws), st, 1));
 }

@@ -195,8 +195,10 @@ __global__ void __launch_bounds__(kThreads, 2)
   const SGeo g = split_geo(p, unit, (int)rank);
   const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
   ptx::cluster_arrive_relaxed();   // phase 0: every CTA of the cluster is running
-  pdl_launch_dependents();
   pdl_wait();   // inputs may come from the kernel before (launched with PDL)
+  // only then may the next kernel be scheduled: the compaction that follows
+  // in e2s_prune copies rows before its own wait
+  pdl_launch_dependents();
   if (p.counters != nullptr && blockIdx.x == 0)
     for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
       p.counters[i] = 0u;

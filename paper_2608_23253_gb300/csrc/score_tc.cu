@@ -143,8 +143,10 @@ __global__ void __launch_bounds__(kThreads, 2)
   const uint32_t rank = ptx::cluster_ctarank();
   const int ncs = p.hpc * p.ntp_max;
   const uint32_t q_half = (uint32_t)ncs * 128u;
-  pdl_launch_dependents();
   pdl_wait();   // inputs may come from the kernel before (launched with PDL)
+  // only then may the next kernel be scheduled: the compaction that follows
+  // in e2s_prune copies rows before its own wait
+  pdl_launch_dependents();
   if (p.counters != nullptr && blockIdx.x == 0)
     for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
       p.counters[i] = 0u;

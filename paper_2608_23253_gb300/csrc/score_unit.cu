@@ -195,8 +195,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t q_half = (uint32_t)p.ntp_max * 128u;
   const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
-  pdl_launch_dependents();   // every CTA is resident: the next kernel may be scheduled
   pdl_wait();   // inputs may come from the kernel before (launched with PDL)
+  // only then may the next kernel be scheduled: the compaction that follows
+  // in e2s_prune copies rows before its own wait
+  pdl_launch_dependents();   // every CTA is resident: the next kernel may be scheduled
   if (p.counters != nullptr && blockIdx.x == 0)
     for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
       p.counters[i] = 0u;
@@ -499,8 +501,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t q_half = (uint32_t)p.ntg * 128u;
   const bool causal = p.mode == E2S_SCORE_CAUSAL_PROB;
-  pdl_launch_dependents();   // every CTA is resident: the next kernel may be scheduled
   pdl_wait();   // inputs may come from the kernel before (launched with PDL)
+  // only then may the next kernel be scheduled: the compaction that follows
+  // in e2s_prune copies rows before its own wait
+  pdl_launch_dependents();   // every CTA is resident: the next kernel may be scheduled
   if (p.counters != nullptr && blockIdx.x == 0)
     for (int i = threadIdx.x; i < la.B * kDecideWordsPerImage; i += blockDim.x)
       p.counters[i] = 0u;
