@@ -76,7 +76,7 @@ WORKLOADS = {
 KERNEL_SOURCES = ("score_split.cu", "sm100_ptx.cuh", "device_common.cuh")
 NCU_TRAFFIC = {
     "cfg1": {"stage": "score", "kernel": "score_split_kernel", "src": KERNEL_SOURCES,
-             "sha": "35c56e8a43f2f801", "bytes": 18227200},
+             "sha": "40a098b0753ae1ac", "bytes": 18227456},
 }
 
 
@@ -91,14 +91,14 @@ ABLATIONS = {"A1": ("vanilla: q = mean attention, no novelty", 16),
 # (profiles/score_*_kernel_*.md), with the source hash they were taken on.
 STREAM_SOURCES = ("score_stream.cu", "sm100_ptx.cuh", "device_common.cuh")
 NCU_TENSOR_PIPE = {
-    "cfg1": {"kernel": "score_split_kernel", "src": KERNEL_SOURCES, "sha": "35c56e8a43f2f801",
-             "pct": 14.15, "profile": "profiles/score_split_kernel_llava_b1.md"},
-    "cfg2": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "a05d629d649c0906",
-             "pct": 26.76, "profile": "profiles/score_stream_kernel_llava_b32.md"},
-    "cfg3": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "a05d629d649c0906",
-             "pct": 31.66, "profile": "profiles/score_stream_kernel_qwen2vl_b16.md"},
-    "cfg4": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "a05d629d649c0906",
-             "pct": 36.57, "profile": "profiles/score_stream_kernel_highres_b8.md"},
+    "cfg1": {"kernel": "score_split_kernel", "src": KERNEL_SOURCES, "sha": "40a098b0753ae1ac",
+             "pct": 15.26, "profile": "profiles/score_split_kernel_llava_b1.md"},
+    "cfg2": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "9348efab60782b02",
+             "pct": 26.85, "profile": "profiles/score_stream_kernel_llava_b32.md"},
+    "cfg3": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "9348efab60782b02",
+             "pct": 31.64, "profile": "profiles/score_stream_kernel_qwen2vl_b16.md"},
+    "cfg4": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "9348efab60782b02",
+             "pct": 36.69, "profile": "profiles/score_stream_kernel_highres_b8.md"},
 }
 
 
