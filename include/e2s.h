@@ -231,13 +231,18 @@ e2s_status e2s_decide_lse(const e2s_layout* layout, const e2s_params* params,
 
 /* One complete pruning step: e2s_decide followed by e2s_compact, three
  * launches (Algorithm 1, one pruning layer; Sec. 3.1 and 4.1-4.3).  Arguments
- * are those of the two calls.  Because the score kernel starts only after all
- * earlier work on the stream, the compaction copies the system and text rows
- * (which do not depend on the selection) while the decision is still running
- * and waits only before the kept visual rows.  The src tensors, keep_count
- * and keep_off must therefore be written by earlier work on the same stream
- * (or be complete before the call), and nothing else may write them while
- * the call runs.  Results are identical to e2s_decide then e2s_compact. */
+ * are those of the two calls.  The score kernel is launched with programmatic
+ * dependence on the kernel before it on the stream: its blocks may be
+ * scheduled while that kernel finishes, but they wait for its completion
+ * before touching memory, and only then let the decision and the compaction
+ * be scheduled.  So all earlier work on the stream is complete before the
+ * compaction copies the system and text rows (which do not depend on the
+ * selection) while the decision is still running; it waits only before the
+ * kept visual rows.  The src tensors, keep_count and keep_off must therefore
+ * be written by earlier work on the same stream (or be complete before the
+ * call), and nothing else may write them while the call runs.  Give it
+ * device-memory sources (it prefetches every candidate row into L2 on small
+ * batches).  Results are identical to e2s_decide then e2s_compact. */
 e2s_status e2s_prune(const e2s_layout* layout, const e2s_params* params,
                      const void* q_text, int64_t q_row_stride,
                      const void* k, int64_t k_row_stride,
