@@ -989,7 +989,7 @@ def run_ours(args, world, rank, local):
             "note": "decision = e2s_decide graph (score + evidence/fusion/Top-K), L2 flushed; "
                     "layer = one LLaMA-2-7B decoder layer in torch bf16 at the same sequence "
                     "length with random weights: sdpa_graph = SDPA causal attention, the whole "
-                    "layer one CUDA graph (the target is judged on this one); eager = fp32 "
+                    "layer one CUDA graph (the < 5 % target refers to this one); eager = fp32 "
                     "attention matrix; est = its FLOPs at the measured sustained bf16 peak"}
         # Table 2 ablations as timed modes, on the same inputs
         abl = {}
