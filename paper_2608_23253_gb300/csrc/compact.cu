@@ -217,15 +217,23 @@ cudaError_t launch_compact(const LayoutArgs& la, const int32_t* keep_idx, const 
   long long blocks = (pairs + warps_per_block - 1) / warps_per_block;
   blocks = std::min<long long>(blocks, (long long)sm_count() * 16);
   const dim3 grid((unsigned)std::max<long long>(blocks, 1));
-  // 8 KiB of a row per warp (112 registers, two CTAs per SM) when there are
-  // only a few rows per warp slot and nothing overlaps the copy; otherwise
-  // 4 KiB per warp (66 registers, three CTAs per SM), which measured faster
-  // in the whole step and on large batches
+  // 16-byte vectors per lane in flight, measured per case: all 16 (8 KiB of a
+  // row per warp) when a standalone call has only a few rows per warp slot;
+  // 8 when the kept rows come out of L2 after the prefetch (the batch-1
+  // step, where the copies after the wait are on the critical path); 2
+  // otherwise -- fewer registers, more resident warps, which measured faster
+  // on every large gather (LLaVA batch 32 step 285.5 -> 278.7 us, Qwen2-VL
+  // batch 16 103.0 -> 97.8 us) while 2 on the prefetched batch-1 step measured
+  // 23.4 -> 26.3 us and 1 slower everywhere
   if (!early && pairs <= (long long)sm_count() * 64)
     return launch_kernel(compact_kernel<16>, grid, dim3(kCompactThreads), 0, st, 0, true, la,
                          keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, early,
                          prefetch);
-  return launch_kernel(compact_kernel<8>, grid, dim3(kCompactThreads), 0, st, 0, true, la,
+  if (prefetch)
+    return launch_kernel(compact_kernel<8>, grid, dim3(kCompactThreads), 0, st, 0, true, la,
+                         keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, early,
+                         prefetch);
+  return launch_kernel(compact_kernel<2>, grid, dim3(kCompactThreads), 0, st, 0, true, la,
                        keep_idx, keep_off, n_tensors, ts, pos_ids, total_rows, status, early,
                        prefetch);
 }
