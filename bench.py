@@ -93,11 +93,11 @@ STREAM_SOURCES = ("score_stream.cu", "sm100_ptx.cuh", "device_common.cuh")
 NCU_TENSOR_PIPE = {
     "cfg1": {"kernel": "score_split_kernel", "src": KERNEL_SOURCES, "sha": "40a098b0753ae1ac",
              "pct": 15.26, "profile": "profiles/score_split_kernel_llava_b1.md"},
-    "cfg2": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "9348efab60782b02",
+    "cfg2": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "86939f0c6763243d",
              "pct": 26.85, "profile": "profiles/score_stream_kernel_llava_b32.md"},
-    "cfg3": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "9348efab60782b02",
+    "cfg3": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "86939f0c6763243d",
              "pct": 31.64, "profile": "profiles/score_stream_kernel_qwen2vl_b16.md"},
-    "cfg4": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "9348efab60782b02",
+    "cfg4": {"kernel": "score_stream_kernel", "src": STREAM_SOURCES, "sha": "86939f0c6763243d",
              "pct": 36.69, "profile": "profiles/score_stream_kernel_highres_b8.md"},
 }
 

@@ -26,7 +26,14 @@
 // K tiles stream through a ring of as many stages as shared memory holds
 // (TMA producer warp; deep enough to cover the load latency), the accumulator
 // is double-buffered in TMEM (MMA warp), so loads, MMAs and the epilogue of
-// consecutive tiles overlap.
+// consecutive tiles overlap.  Short units (under 24 key tiles on average)
+// get a second query buffer in place of a ring stage, so the next unit's
+// queries are in before the current unit ends.  With fewer than 16 units per
+// CTA the units come from a counter in the workspace, handed by the producer
+// to the other roles through a small shared-memory ring (heaviest images
+// first below 6 units per CTA); otherwise they go round-robin.  In batches of
+// mixed text length the units of at most 64 rows still run split.  Every
+// image's layout is staged in shared memory once per CTA.
 //
 // Warp roles (608 threads): warp 0 TMA producer, warp 1 TMEM allocator and MMA
 // issuer of the even tiles, warp 18 MMA issuer of the odd tiles, warps 2-17
